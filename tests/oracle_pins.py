@@ -1,0 +1,285 @@
+"""Pins for the fp64 oracle: facts fixed by the paper or by mathematics.
+
+Each check takes an oracle object (oracle.Oracle) and raises AssertionError if
+the oracle disagrees with the fact.  test_oracle_pins.py runs them against the
+real oracle; test_oracle_mutants.py runs them against deliberately broken
+copies of the oracle to show that each plausible mistake fails at least one
+pin.  None of these checks re-types the oracle's own formula: they use values
+printed in the paper, closed forms, invariants and an independent 50-digit
+decimal brute force.
+"""
+from __future__ import annotations
+
+import decimal
+import math
+
+import numpy as np
+
+from conftest import load_golden
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+def _f32(x):
+    return np.asarray(x, dtype=np.float32)
+
+
+# ----------------------------------------------------------------------------------------------
+# 1. The paper's worked example (Section 5, Tables tab:attn_weights and tab:output; Appendix A)
+# ----------------------------------------------------------------------------------------------
+def pin_paper_example(o):
+    g = load_golden("paper_example_n3_d4.txt")
+    Q, K, V = _f32(g["Q"]), _f32(g["K"]), _f32(g["V"])
+    w, out = o.weights(Q, K, V, 0.5)
+    # Printed to 4 decimals from inputs that were themselves printed to 4 decimals.
+    assert np.max(np.abs(w - g["W"])) <= 2e-4, w
+    assert np.max(np.abs(out - g["O"])) <= 2e-4, out
+    assert np.max(np.abs(w.sum(axis=1) - 1.0)) <= 1e-12
+    # Appendix A, row 0: scaled scores x, z = x - max x, e^z and their sum.
+    x0 = o.scores(Q, K, 0.5)[0]
+    assert np.max(np.abs(x0 - g["X0"][0])) <= 2e-4, x0
+    z0 = x0 - x0.max()
+    assert np.max(np.abs(z0 - g["Z0"][0])) <= 2e-4
+    # e^z and Z follow from the oracle's weights: w = e^z / Z with max e^z = 1.
+    e0 = w[0] / w[0].max()
+    assert np.max(np.abs(e0 - g["E0"][0])) <= 2e-4, e0
+    assert abs(1.0 / w[0].max() - g["DEN0"][0, 0]) <= 2e-4
+
+
+# ----------------------------------------------------------------------------------------------
+# 2. Independent brute force: 50-digit decimal arithmetic on tiny inputs
+# ----------------------------------------------------------------------------------------------
+def decimal_attention(Q, K, V, scale):
+    """softmax(scale Q K^T) V evaluated in 50-digit decimal arithmetic (no max shift needed)."""
+    ctx = decimal.Context(prec=50)
+    D = lambda x: decimal.Decimal(float(x))
+    n, dk = Q.shape
+    nk, dv = V.shape
+    sc = D(scale)
+    out = np.zeros((n, dv))
+    for i in range(n):
+        ex = []
+        for k in range(nk):
+            s = decimal.Decimal(0)
+            for j in range(dk):
+                s = ctx.add(s, ctx.multiply(D(Q[i, j]), D(K[k, j])))
+            ex.append(ctx.exp(ctx.multiply(s, sc)))
+        tot = decimal.Decimal(0)
+        for e in ex:
+            tot = ctx.add(tot, e)
+        for c in range(dv):
+            acc = decimal.Decimal(0)
+            for k in range(nk):
+                acc = ctx.add(acc, ctx.multiply(ctx.divide(ex[k], tot), D(V[k, c])))
+            out[i, c] = float(acc)
+    return out
+
+
+def pin_decimal_bruteforce(o):
+    shapes = [(1, 1, 1, 1), (2, 3, 4, 5), (5, 7, 3, 2), (8, 8, 8, 8), (3, 6, 8, 1)]
+    for t, (nq, nk, dk, dv) in enumerate(shapes):
+        r = _rng(100 + t)
+        Q = _f32(r.normal(size=(nq, dk)) * 2.0)
+        K = _f32(r.normal(size=(nk, dk)))
+        V = _f32(r.normal(size=(nk, dv)))
+        scale = 1.0 / math.sqrt(dk)
+        ref = decimal_attention(Q, K, V, scale)
+        got = o.attn(Q, K, V, scale)
+        err = np.max(np.abs(got - ref)) / max(1e-300, np.max(np.abs(ref)))
+        assert err <= 1e-13, (nq, nk, dk, dv, err)
+
+
+# ----------------------------------------------------------------------------------------------
+# 3. Invariants and closed forms
+# ----------------------------------------------------------------------------------------------
+def pin_row_sums(o):
+    for t, (nq, nk, dk) in enumerate([(7, 13, 5), (16, 300, 64), (3, 1, 8)]):
+        r = _rng(200 + t)
+        Q = _f32(r.normal(size=(nq, dk)) * 3)
+        K = _f32(r.normal(size=(nk, dk)))
+        V = _f32(r.normal(size=(nk, 4)))
+        w, _ = o.weights(Q, K, V, 1.0 / math.sqrt(dk))
+        assert np.all(w >= 0.0)
+        assert np.max(np.abs(w.sum(axis=1) - 1.0)) <= nk * 1e-15 + 1e-15
+
+
+def pin_v_ones(o):
+    r = _rng(300)
+    Q = _f32(r.normal(size=(2, 3, 33, 16)) * 4)
+    K = _f32(r.normal(size=(2, 3, 71, 16)))
+    V = np.ones((2, 3, 71, 8), dtype=np.float32)
+    out = o.attn(Q, K, V, 0.25)
+    assert np.max(np.abs(out - 1.0)) <= 1e-14
+
+
+def pin_q_zero_column_mean(o):
+    r = _rng(301)
+    K = _f32(r.normal(size=(1, 2, 50, 8)))
+    V = _f32(r.normal(size=(1, 2, 50, 6)))
+    Q = np.zeros((1, 2, 9, 8), dtype=np.float32)
+    mean = V.astype(np.float64).mean(axis=2, keepdims=True)
+    out = o.attn(Q, K, V, 0.3)
+    assert np.max(np.abs(out - mean)) <= 1e-14
+    # scale = 0 gives the same, for any Q.
+    Q2 = _f32(r.normal(size=(1, 2, 9, 8)))
+    out2 = o.attn(Q2, K, V, 0.0)
+    assert np.max(np.abs(out2 - mean)) <= 1e-14
+
+
+def pin_single_key(o):
+    r = _rng(302)
+    Q = _f32(r.normal(size=(2, 2, 5, 8)) * 10)
+    K = _f32(r.normal(size=(2, 2, 1, 8)))
+    V = _f32(r.normal(size=(2, 2, 1, 3)))
+    out = o.attn(Q, K, V, 0.7)
+    assert np.array_equal(out, np.broadcast_to(V.astype(np.float64), out.shape))
+
+
+def pin_two_keys_logistic(o):
+    """Two keys: O = V0 + sigmoid(s1 - s0) (V1 - V0), with s_k = scale <q, k_k>."""
+    r = _rng(303)
+    Q = _f32(r.normal(size=(11, 6)))
+    K = _f32(r.normal(size=(2, 6)))
+    V = _f32(r.normal(size=(2, 5)))
+    scale = 0.9
+    q64, k64, v64 = Q.astype(np.float64), K.astype(np.float64), V.astype(np.float64)
+    d = scale * (q64 @ k64[1] - q64 @ k64[0])
+    sig = 1.0 / (1.0 + np.exp(-d))
+    ref = v64[0][None, :] + sig[:, None] * (v64[1] - v64[0])[None, :]
+    out = o.attn(Q, K, V, scale)
+    assert np.max(np.abs(out - ref)) <= 1e-14
+
+
+def pin_convexity(o):
+    r = _rng(304)
+    Q = _f32(r.normal(size=(1, 1, 40, 12)) * 5)
+    K = _f32(r.normal(size=(1, 1, 90, 12)))
+    V = _f32(r.normal(size=(1, 1, 90, 7)))
+    out = o.attn(Q, K, V, 1.0 / math.sqrt(12))[0, 0]
+    lo = V[0, 0].min(axis=0).astype(np.float64)
+    hi = V[0, 0].max(axis=0).astype(np.float64)
+    assert np.all(out >= lo[None, :] - 1e-15) and np.all(out <= hi[None, :] + 1e-15)
+
+
+def pin_key_permutation_and_row_locality(o):
+    r = _rng(305)
+    Q = _f32(r.normal(size=(2, 2, 20, 8)))
+    K = _f32(r.normal(size=(2, 2, 37, 8)))
+    V = _f32(r.normal(size=(2, 2, 37, 5)))
+    base = o.attn(Q, K, V, 0.35)
+    perm = r.permutation(37)
+    permd = o.attn(Q, K[:, :, perm], V[:, :, perm], 0.35)
+    assert np.max(np.abs(permd - base)) <= 1e-14
+    # Output row i depends on query row i only (and heads are independent).
+    Q2 = Q.copy()
+    Q2[1, 0, 3] = _f32(r.normal(size=8))
+    changed = o.attn(Q2, K, V, 0.35)
+    mask = np.ones(base.shape[:3], dtype=bool)
+    mask[1, 0, 3] = False
+    assert np.array_equal(changed[mask], base[mask])
+    assert not np.array_equal(changed[1, 0, 3], base[1, 0, 3])
+    # Rows of a query matrix flipped upside down give the output flipped the same way.
+    flipped = o.attn(Q[:, :, ::-1], K, V, 0.35)
+    assert np.array_equal(flipped, base[:, :, ::-1])
+
+
+def pin_head_independence(o):
+    """Each (b,h) slice is its own 2-D problem (Remark in Section 4.2)."""
+    r = _rng(306)
+    Q = _f32(r.normal(size=(2, 3, 9, 8)))
+    K = _f32(r.normal(size=(2, 3, 14, 8)))
+    V = _f32(r.normal(size=(2, 3, 14, 4)))
+    full = o.attn(Q, K, V, 0.5)
+    for b in range(2):
+        for h in range(3):
+            one = o.attn(Q[b, h], K[b, h], V[b, h], 0.5)
+            assert np.array_equal(one, full[b, h])
+
+
+def pin_shift_invariance(o):
+    """Adding a constant to a score row leaves the output unchanged (Eq. stable_softmax)."""
+    r = _rng(307)
+    Q = _f32(r.normal(size=(1, 2, 10, 16)) * 2)
+    K = _f32(r.normal(size=(1, 2, 33, 16)))
+    V = _f32(r.normal(size=(1, 2, 33, 4)))
+    base = o.attn(Q, K, V, 0.25)
+    for c in (-1e3, 0.5, 1e3):
+        sh = np.full(20, c)
+        out = o.attn_shifted(Q, K, V, 0.25, sh)
+        assert np.max(np.abs(out - base)) <= 1e-11, c
+    # The same through the inputs: K[..,0] = 1 and Q[..,0] = delta adds scale*delta to row i.
+    K2 = K.copy()
+    K2[..., 0] = 1.0
+    Qa = Q.copy()
+    Qa[..., 0] = 0.0
+    Qb = Qa.copy()
+    Qb[..., 0] = _f32(r.integers(-64, 64, size=Qb.shape[:3]))
+    a = o.attn(Qa, K2, V, 0.25)
+    b = o.attn(Qb, K2, V, 0.25)
+    assert np.max(np.abs(a - b)) <= 1e-12
+
+
+def pin_large_scores_stable(o):
+    """Scores of magnitude far beyond exp's range: max subtraction keeps them finite."""
+    r = _rng(308)
+    Q = _f32(r.normal(size=(1, 1, 6, 32)) * 40)
+    K = _f32(r.normal(size=(1, 1, 25, 32)) * 40)
+    V = _f32(r.normal(size=(1, 1, 25, 3)))
+    s = o.scores(Q, K, 1.0)
+    assert np.max(np.abs(s)) > 2000  # exp() of these would overflow without the shift
+    out = o.attn(Q, K, V, 1.0)
+    assert np.all(np.isfinite(out))
+    # With such a spread, the softmax is one-hot on each row's arg-max key.
+    top = np.argmax(s[0, 0], axis=1)
+    srt = np.sort(s[0, 0], axis=1)
+    assert np.all(srt[:, -1] - srt[:, -2] > 40)
+    assert np.max(np.abs(out[0, 0] - V[0, 0][top].astype(np.float64))) <= 1e-15
+
+
+def pin_planted_rows(o):
+    """Q[i] := K[k*] with a margin > 30 over the next score gives O[i] = V[k*] (exp(-30) ~ 1e-13)."""
+    r = _rng(309)
+    K = _f32(r.normal(size=(1, 1, 64, 128)) * 8)
+    V = _f32(r.normal(size=(1, 1, 64, 5)))
+    Q = _f32(r.normal(size=(1, 1, 8, 128)) * 8)
+    Q[0, 0, 3] = K[0, 0, 17]
+    scale = 1.0 / math.sqrt(128)
+    s = o.scores(Q, K, scale)[0, 0, 3]
+    srt = np.sort(s)
+    assert srt[-1] - srt[-2] > 30 and np.argmax(s) == 17
+    out = o.attn(Q, K, V, scale)
+    assert np.max(np.abs(out[0, 0, 3] - V[0, 0, 17])) <= 1e-12
+
+
+def pin_rows_and_threads(o):
+    """Sampled rows equal the full computation, and thread count does not change any bit."""
+    r = _rng(310)
+    Q = _f32(r.normal(size=(2, 2, 30, 16)))
+    K = _f32(r.normal(size=(2, 2, 45, 16)))
+    V = _f32(r.normal(size=(2, 2, 45, 8)))
+    full1 = o.attn(Q, K, V, 0.25, nthreads=1)
+    full4 = o.attn(Q, K, V, 0.25, nthreads=4)
+    assert np.array_equal(full1, full4)
+    rows = np.array([0, 29, 30, 77, 119])
+    got = o.rows(Q, K, V, 0.25, rows)
+    assert np.array_equal(got, full1.reshape(-1, 8)[rows])
+
+
+ALL_PINS = [
+    pin_paper_example,
+    pin_decimal_bruteforce,
+    pin_row_sums,
+    pin_v_ones,
+    pin_q_zero_column_mean,
+    pin_single_key,
+    pin_two_keys_logistic,
+    pin_convexity,
+    pin_key_permutation_and_row_locality,
+    pin_head_independence,
+    pin_shift_invariance,
+    pin_large_scores_stable,
+    pin_planted_rows,
+    pin_rows_and_threads,
+]
