@@ -1,0 +1,136 @@
+/*
+ * moa_attn: forward pass of scaled dot-product attention on sm_103a (GB300),
+ * computed in the paper's Denotational Normal Form: no score, probability or
+ * transposed-K array ever exists in device memory, so Q, K and V are read once
+ * and O is written once.
+ *
+ * Paper: "Attention at the Theoretical Minimum: A Mathematics of Arrays
+ * Framework for Memory-Optimal Transformer Kernels" (Mullin, Hains).
+ *
+ * Shared library: libmoa_attn.so (plain C ABI, no C++ or PyTorch types).
+ * Every entry point is thread-safe; moa_last_error() is per calling thread.
+ */
+#ifndef MOA_ATTN_H
+#define MOA_ATTN_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Element types of Q, K, V and O (all four share one type). */
+enum moa_dtype {
+    MOA_FP32 = 0, /* IEEE binary32; computed on CUDA cores in fp32 (no TF32) */
+    MOA_BF16 = 1  /* bfloat16; tensor-core products, fp32 accumulation and softmax */
+};
+
+/* Status codes returned by every int-valued entry point. */
+enum moa_status {
+    MOA_OK = 0,
+    MOA_ERR_INVALID_ARG = 1,       /* null pointer, a size <= 0, non-finite scale, O overlaps an input */
+    MOA_ERR_UNSUPPORTED_DTYPE = 2, /* dtype is not one of enum moa_dtype */
+    MOA_ERR_UNSUPPORTED_SHAPE = 3, /* head dimensions or sizes outside what the kernels take */
+    MOA_ERR_MISALIGNED = 4,        /* a pointer not 16-byte aligned, or a row not a multiple of 16 bytes */
+    MOA_ERR_CUDA = 5,              /* a CUDA runtime/driver call failed (message in moa_last_error) */
+    MOA_ERR_DEVICE_TIMEOUT = 6     /* a kernel gave up on a wait and recorded it in the status word */
+};
+
+/*
+ * moa_attn_fwd -- O = softmax(scale * Q K^T) V, one independent problem per (b, h).
+ *
+ * Defines: paper Section 4.1, Eq. (attention) with the max-subtracted softmax of
+ * Eq. (stable_softmax) and the contraction with V of Eq. (output_dnf), computed
+ * per (batch, head) slice as in the Remark of Section 4.2 (Eq. batched_mm).
+ * For every b < B, h < H, i < N_q, c < d_v:
+ *     s_k        = scale * sum_{j < d_k} Q[b,h,i,j] * K[b,h,k,j]      (k < N_k)
+ *     O[b,h,i,c] = sum_k exp(s_k - max_k' s_k') / (sum_k'' exp(s_k'' - max_k' s_k')) * V[b,h,k,c]
+ * The softmax runs over the key axis N_k; N_q and N_k may differ, as may d_k
+ * and d_v.  No mask, dropout or bias.
+ *
+ * Arguments:
+ *   Q  device pointer, [B, H, N_q, d_k], contiguous row-major, element type dtype (read only)
+ *   K  device pointer, [B, H, N_k, d_k], same layout, read as stored (no transpose copy)
+ *   V  device pointer, [B, H, N_k, d_v], same layout
+ *   O  device pointer, [B, H, N_q, d_v], same element type; written, must not overlap Q, K, V
+ *   B, H, N_q, N_k, d_k, d_v   sizes, each >= 1
+ *   scale   multiplier of the scores, any finite value (the paper uses 1/sqrt(d_k))
+ *   dtype   MOA_FP32 or MOA_BF16
+ *   stream  a cudaStream_t (NULL = legacy default stream) of the current device
+ *
+ * Supported sizes:
+ *   MOA_BF16: d_k, d_v in {64, 128}; N_q, N_k < 2^31; B*H < 2^31.
+ *   MOA_FP32: 1 <= d_k, d_v <= 128 and d_k, d_v multiples of 4.
+ * Alignment: Q, K, V, O 16-byte aligned.
+ *
+ * Ownership and memory: the caller owns all four buffers.  The call allocates
+ * no device memory and uses no workspace; the kernels keep every intermediate
+ * (scores, probabilities, running max and sum) in registers, shared memory and
+ * tensor memory.
+ *
+ * Behaviour: asynchronous on `stream`; returns after the launch.  Arguments
+ * are checked before anything is launched; on a non-OK return nothing was
+ * launched and moa_last_error() describes the problem.  Kernel waits are
+ * bounded: a wait that runs out records MOA_ERR_DEVICE_TIMEOUT in a device
+ * status word (see moa_get_device_status) and the kernel returns early.
+ */
+int moa_attn_fwd(const void* Q, const void* K, const void* V, void* O, int64_t B, int64_t H,
+                 int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v, float scale, int dtype,
+                 void* stream);
+
+/*
+ * moa_attn_fwd_staged -- the same computation with host-resident inputs and output.
+ *
+ * Defines: as moa_attn_fwd (paper Section 4.1, Eq. attention).  Copies hQ, hK,
+ * hV (host memory, ideally page-locked) into the caller's device buffers dQ,
+ * dK, dV, runs moa_attn_fwd on them and copies dO back into hO, all enqueued
+ * on `stream` in that order.  Sizes, layouts, dtype and alignment rules are
+ * those of moa_attn_fwd; d* are device pointers owned by the caller, h* host
+ * pointers owned by the caller.  Asynchronous: hO holds the result once
+ * `stream` has been synchronised.  Allocates nothing.
+ */
+int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO, void* dQ,
+                        void* dK, void* dV, void* dO, int64_t B, int64_t H, int64_t N_q,
+                        int64_t N_k, int64_t d_k, int64_t d_v, float scale, int dtype,
+                        void* stream);
+
+/*
+ * moa_last_error -- human-readable reason for the last non-OK status returned
+ * on the calling thread ("" if none).  The string is owned by the library and
+ * stays valid until the next call on the same thread.
+ */
+const char* moa_last_error(void);
+
+/*
+ * moa_get_device_status -- synchronises `stream`, then returns and clears the
+ * device status word that bounded waits write on timeout: MOA_OK if no kernel
+ * timed out since the last call, MOA_ERR_DEVICE_TIMEOUT otherwise,
+ * MOA_ERR_CUDA if the synchronisation itself failed.
+ */
+int moa_get_device_status(void* stream);
+
+/*
+ * moa_attn_flops -- floating-point operations of the two contractions,
+ * 2*B*H*N_q*N_k*(d_k + d_v): the two matrix products of Eq. (attention),
+ * Q K^T and the product of the weights with V (exponentials, maxima and the
+ * division are not counted).
+ */
+double moa_attn_flops(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v);
+
+/*
+ * moa_attn_dnf_bytes -- the memory-traffic lower bound of the paper (Theorem
+ * lower_bound, Section 6.5): read Q, K, V once and write O once,
+ *     elt * B * H * (N_q*d_k + N_k*d_k + N_k*d_v + N_q*d_v)
+ * with elt = 4 (MOA_FP32) or 2 (MOA_BF16); returns -1 for an unknown dtype.
+ */
+double moa_attn_dnf_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int64_t d_k,
+                          int64_t d_v, int dtype);
+
+/* moa_attn_version -- library version, major*10000 + minor*100 + patch. */
+int moa_attn_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MOA_ATTN_H */

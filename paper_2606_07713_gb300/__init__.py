@@ -1,0 +1,109 @@
+"""DNF attention forward for GB300 (sm_103a).
+
+O = softmax(scale * Q K^T) V with a max-subtracted softmax, computed without any
+score, probability or transposed-K array in device memory (the Denotational
+Normal Form of Mullin & Hains, "Attention at the Theoretical Minimum").
+
+The computation runs in libmoa_attn.so (hand-written CUDA: a tcgen05/TMEM/TMA
+kernel for bf16 and a CUDA-core kernel for fp32).  This package is its thin
+Python binding: PyTorch supplies device memory and the current stream, nothing
+else.  There is no CPU fallback.
+"""
+from __future__ import annotations
+
+import math
+
+from ._lib import (MOA_BF16, MOA_FP32, MoaError, check, lib, moa_attn_dnf_bytes,  # noqa: F401
+                   moa_attn_flops, moa_attn_fwd, moa_attn_fwd_staged, moa_attn_version,
+                   moa_get_device_status, moa_last_error)
+
+__all__ = ["attn_fwd", "attn_fwd_staged", "get_device_status", "attn_flops", "dnf_bytes",
+           "MOA_FP32", "MOA_BF16", "MoaError", "moa_attn_fwd", "moa_attn_fwd_staged",
+           "moa_last_error", "moa_get_device_status", "moa_attn_flops", "moa_attn_dnf_bytes",
+           "moa_attn_version"]
+
+
+def _dtype_code(t) -> int:
+    import torch
+    if t.dtype == torch.bfloat16:
+        return MOA_BF16
+    if t.dtype == torch.float32:
+        return MOA_FP32
+    raise TypeError(f"unsupported dtype {t.dtype}; use torch.bfloat16 or torch.float32")
+
+
+def _dims(q, k, v):
+    if q.dim() != 4 or k.dim() != 4 or v.dim() != 4:
+        raise ValueError("q, k, v must be [B, H, N, d]")
+    B, H, Nq, dk = q.shape
+    if tuple(k.shape[:2]) != (B, H) or tuple(v.shape[:2]) != (B, H):
+        raise ValueError(f"batch/head mismatch: {tuple(q.shape)} {tuple(k.shape)} {tuple(v.shape)}")
+    if k.shape[3] != dk or v.shape[2] != k.shape[2]:
+        raise ValueError(f"shape mismatch: {tuple(q.shape)} {tuple(k.shape)} {tuple(v.shape)}")
+    return B, H, Nq, k.shape[2], dk, v.shape[3]
+
+
+def attn_fwd(q, k, v, scale: float | None = None, out=None, stream=None):
+    """O = softmax(scale * q k^T) v for CUDA tensors [B, H, N, d] (bf16 or fp32).
+
+    scale defaults to 1/sqrt(d_k).  Runs asynchronously on `stream` (default:
+    torch's current stream of q's device) and returns `out` (allocated if None).
+    """
+    import torch
+    for t in (q, k, v):
+        if not t.is_cuda:
+            raise ValueError("attn_fwd needs CUDA tensors")
+        if not t.is_contiguous():
+            raise ValueError("attn_fwd needs contiguous tensors")
+    if not (q.dtype == k.dtype == v.dtype):
+        raise TypeError("q, k, v must share one dtype")
+    code = _dtype_code(q)
+    B, H, Nq, Nk, dk, dv = _dims(q, k, v)
+    if scale is None:
+        scale = 1.0 / math.sqrt(dk)
+    if out is None:
+        out = torch.empty((B, H, Nq, dv), dtype=q.dtype, device=q.device)
+    elif out.shape != (B, H, Nq, dv) or out.dtype != q.dtype or not out.is_contiguous():
+        raise ValueError("out has the wrong shape, dtype or layout")
+    with torch.cuda.device(q.device):
+        s = stream if stream is not None else torch.cuda.current_stream(q.device)
+        check(moa_attn_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), B, H, Nq, Nk,
+                           dk, dv, float(scale), code, s.cuda_stream))
+    return out
+
+
+def attn_fwd_staged(hq, hk, hv, ho, dq, dk_, dv_, do, scale: float | None = None, stream=None):
+    """Host tensors in, host tensor out: copies hq/hk/hv to the device buffers dq/dk_/dv_,
+    runs the kernel into do and copies it back into ho, all on one stream.  The result is in
+    ho after the stream is synchronised."""
+    import torch
+    code = _dtype_code(dq)
+    B, H, Nq, Nk, dk, dv = _dims(dq, dk_, dv_)
+    for h, d in ((hq, dq), (hk, dk_), (hv, dv_), (ho, do)):
+        if h.is_cuda or not d.is_cuda or h.shape != d.shape or h.dtype != d.dtype:
+            raise ValueError("staged call needs matching host and device tensors")
+        if not (h.is_contiguous() and d.is_contiguous()):
+            raise ValueError("staged call needs contiguous tensors")
+    if scale is None:
+        scale = 1.0 / math.sqrt(dk)
+    with torch.cuda.device(dq.device):
+        s = stream if stream is not None else torch.cuda.current_stream(dq.device)
+        check(moa_attn_fwd_staged(hq.data_ptr(), hk.data_ptr(), hv.data_ptr(), ho.data_ptr(),
+                                  dq.data_ptr(), dk_.data_ptr(), dv_.data_ptr(), do.data_ptr(),
+                                  B, H, Nq, Nk, dk, dv, float(scale), code, s.cuda_stream))
+    return ho
+
+
+def get_device_status(stream=None) -> int:
+    """Synchronises the stream and returns/clears the kernels' timeout status word."""
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return moa_get_device_status(s.cuda_stream)
+
+
+def attn_flops(B, H, N_q, N_k, d_k, d_v) -> float:
+    return moa_attn_flops(B, H, N_q, N_k, d_k, d_v)
+
+
+def dnf_bytes(B, H, N_q, N_k, d_k, d_v, dtype: int) -> float:
+    return moa_attn_dnf_bytes(B, H, N_q, N_k, d_k, d_v, dtype)

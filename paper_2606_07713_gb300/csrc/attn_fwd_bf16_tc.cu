@@ -1,0 +1,599 @@
+// bf16 attention forward on the fifth-generation tensor cores (tcgen05 + TMEM + TMA), sm_103a.
+//
+// What it computes: O = softmax(scale * Q K^T) V per (b, h) slice (paper Section 4.1,
+// Eq. attention; the slices are the independent 2-D problems of the Remark in Section 4.2).
+// How it keeps the DNF's memory pattern (Section 4, Fig. pipeline): no score matrix, no
+// exponential buffer, no transposed K and no denominator vector exists in global memory.
+//
+//   * Scores S = Q K^T (Eq. mm_psi) are tensor-core products of a Q tile and a K tile, both
+//     read from shared memory in their stored row-major layout (K is the "K-major" B operand,
+//     so no transpose copy exists).  S lands in tensor memory (TMEM) as fp32.
+//   * Step I (row maximum, Section 4.3), Step II (exponentials, Section 4.4) and Step III
+//     (denominator, Section 4.5) run online per row in the registers of one softmax thread:
+//     running maximum m and running sum l over the key tiles.  When the maximum of a new tile
+//     exceeds m by more than kRescaleLog2 (in log2 units), m is raised and O and l are
+//     rescaled by exp2(m_old - m_new); otherwise the stale m is kept.  Both are exact: O and l
+//     always share the same reference maximum, and exponentials stay <= 2^kRescaleLog2.
+//   * The unnormalised probabilities P are rounded to bf16 and written back into the TMEM
+//     columns of S, from where the second tensor-core product O += P V (Eq. output_dnf) reads
+//     them directly.  V is the "MN-major" B operand, again as stored.
+//   * Step IV (division, Section 4.5) is applied once per row in the epilogue: O / l.
+//
+// CTA organisation (one CTA per SM: 512 TMEM columns, ~192 KB shared memory):
+//   work item = (b*H + h, block of 256 query rows) = two 128-row Q tiles;
+//   warps 0-3: softmax + epilogue of Q tile 0; warps 4-7: same for Q tile 1
+//              (thread t of such a warpgroup owns query row t of its tile);
+//   warp 8:    TMEM allocation and the single thread that issues all tcgen05.mma;
+//   warp 9:    the single thread that issues all TMA loads.
+// K and V tiles of 128 keys stream through an NS-stage shared-memory ring in the order
+// K0, V0, K1, V1, ...; the MMA thread issues, per key tile n >= 1 and Q tile j,
+// O_j += P_j(n-1) V(n-1) and then S_j = Q_j K(n)^T, so the tensor core always has the other
+// Q tile's work while one softmax warpgroup runs.
+//
+// TMEM columns: S0 [0,128) S1 [128,256) O0 [256,256+DV) O1 [256+DV, 256+2DV); lane = row.
+//
+// Every mbarrier wait is bounded (globaltimer); on expiry the kernel records
+// MOA_ERR_DEVICE_TIMEOUT in g_moa_bf16_status, makes every role leave its loop, and still
+// frees its TMEM before returning.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdio>
+#include <mutex>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace moa {
+
+__device__ unsigned int g_moa_bf16_status = 0;
+
+namespace {
+
+using namespace ptx;
+
+constexpr int kBM = 128;          // query rows per Q tile (= TMEM lanes)
+constexpr int kBN = 128;          // keys per K/V tile
+constexpr int kQTiles = 2;        // Q tiles per CTA
+constexpr int kThreads = 320;     // 8 softmax warps + MMA warp + TMA warp
+constexpr int kMmaWarp = 8;
+constexpr int kLoadWarp = 9;
+constexpr int kTmemCols = 512;
+constexpr float kRescaleLog2 = 8.0f;  // lazy-rescale threshold: exponentials stay <= 2^8
+
+template <int DK, int DV>
+struct Cfg {
+  static_assert(DK == 64 || DK == 128, "d_k must be 64 or 128");
+  static_assert(DV == 64 || DV == 128, "d_v must be 64 or 128");
+  // One 128-byte swizzle panel holds 64 bf16 columns of 128 rows: 16 KB.
+  static constexpr int kPanelBytes = 128 * 128;
+  static constexpr int kQTileBytes = kBM * DK * 2;
+  static constexpr int kKTileBytes = kBN * DK * 2;
+  static constexpr int kVTileBytes = kBN * DV * 2;
+  static constexpr int kStageBytes = kKTileBytes > kVTileBytes ? kKTileBytes : kVTileBytes;
+  static constexpr int kStages = (DK == 64 && DV == 64) ? 8 : 4;
+  static constexpr int kOffQ = 0;
+  static constexpr int kOffKV = kOffQ + kQTiles * kQTileBytes;
+  static constexpr int kOffBar = kOffKV + kStages * kStageBytes;
+  // barriers: full[NS], empty[NS], q_full, s_full[2], p_ready[2], o_done
+  static constexpr int kNumBars = 2 * kStages + 6;
+  static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
+  static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack for 1024-B alignment
+  static constexpr uint32_t kTmemS0 = 0, kTmemS1 = 128, kTmemO0 = 256, kTmemO1 = 256 + DV;
+  static_assert(kTmemO1 + DV <= kTmemCols, "TMEM budget");
+  static_assert(kSmemBytes <= 232448, "shared memory budget");
+};
+
+// Instruction descriptor of tcgen05.mma kind::f16: D fp32, A and B bf16, dense.
+//   bits 4-5 D format (1 = f32), 7-9 A format (1 = bf16), 10-12 B format (1 = bf16),
+//   15 A major (0 = K-major), 16 B major (1 = MN-major), 17-22 N >> 3, 24-28 M >> 4.
+__host__ __device__ constexpr uint32_t make_idesc(int M, int N, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | ((b_mn_major ? 1u : 0u) << 16) |
+         (uint32_t(N >> 3) << 17) | (uint32_t(M >> 4) << 24);
+}
+
+// Shared-memory matrix descriptor, 128-byte swizzle (layout code 2 in bits 61-63), version 1
+// (bits 46-47).  Start address, leading and stride byte offsets in 16-byte units.
+__device__ __forceinline__ uint64_t make_sdesc_sw128(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+  return uint64_t((addr & 0x3FFFFu) >> 4) | (uint64_t((lbo >> 4) & 0x3FFFu) << 16) |
+         (uint64_t((sbo >> 4) & 0x3FFFu) << 32) | (uint64_t(1) << 46) | (uint64_t(2) << 61);
+}
+
+struct WaitCtl {
+  volatile int* abort_flag;
+  uint64_t limit_ns;
+};
+
+// Bounded mbarrier wait.  Returns false (and raises the CTA abort flag and the global status
+// word) if the phase did not complete within limit_ns, or if another role already aborted.
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, const WaitCtl& w) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 63u) == 0) {
+      if (*w.abort_flag) return false;
+      if (globaltimer_ns() - t0 > w.limit_ns) {
+        *w.abort_flag = 1;
+        atomicExch(&g_moa_bf16_status, 6u);  // MOA_ERR_DEVICE_TIMEOUT
+        return false;
+      }
+    }
+  }
+}
+
+// Time-limited wait that ignores the abort flag: used on the way out so that no TMA copy or
+// tensor-core operation is still writing shared or tensor memory when the CTA exits.
+__device__ __forceinline__ void wait_quiesce(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
+  const uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (globaltimer_ns() - t0 > limit_ns) {
+      atomicExch(&g_moa_bf16_status, 6u);
+      return;
+    }
+  }
+}
+
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);  // .x (low 16 bits) = lo
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Loads 128 fp32 columns of this thread's TMEM lane into s[] and waits for completion.
+__device__ __forceinline__ void tmem_load_row128(uint32_t taddr, uint32_t* s) {
+  tmem_ld_32x32b_x32(taddr + 0, s + 0);
+  tmem_ld_32x32b_x32(taddr + 32, s + 32);
+  tmem_ld_32x32b_x32(taddr + 64, s + 64);
+  tmem_ld_32x32b_x32(taddr + 96, s + 96);
+  tmem_wait_ld();
+  reg_anchor_x32(s + 0);
+  reg_anchor_x32(s + 32);
+  reg_anchor_x32(s + 64);
+  reg_anchor_x32(s + 96);
+}
+
+// Multiplies DV fp32 TMEM columns of this thread's lane by alpha (warp-collective).
+template <int DV>
+__device__ __forceinline__ void tmem_scale_row(uint32_t taddr, float alpha) {
+#pragma unroll
+  for (int c = 0; c < DV; c += 32) {
+    uint32_t o[32];
+    tmem_ld_32x32b_x32(taddr + c, o);
+    tmem_wait_ld();
+    reg_anchor_x32(o);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+    tmem_st_32x32b_x32(taddr + c, o);
+  }
+  tmem_wait_st();
+}
+
+template <int DK, int DV>
+__global__ void __launch_bounds__(kThreads, 1)
+attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
+                        const __grid_constant__ CUtensorMap tmK,
+                        const __grid_constant__ CUtensorMap tmV, __nv_bfloat16* __restrict__ O,
+                        int Nq, int Nk, int n_qblocks, float c_log2, uint64_t wait_limit_ns) {
+  using C = Cfg<DK, DV>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  const uint32_t sQ = smem_u32(smem + C::kOffQ);
+  const uint32_t sKV = smem_u32(smem + C::kOffKV);
+  const uint32_t bar0 = smem_u32(smem + C::kOffBar);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (C::kStages + s); };
+  const uint32_t q_full = bar0 + 8u * (2 * C::kStages);
+  auto s_full = [&](int j) { return bar0 + 8u * (2 * C::kStages + 1 + j); };
+  auto p_ready = [&](int j) { return bar0 + 8u * (2 * C::kStages + 3 + j); };
+  const uint32_t o_done = bar0 + 8u * (2 * C::kStages + 5);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int bh = blockIdx.x / n_qblocks;
+  const int q0 = (blockIdx.x % n_qblocks) * (kQTiles * kBM);
+  const int n_kt = (Nk + kBN - 1) / kBN;
+  const WaitCtl wc{abort_flag, wait_limit_ns};
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    mbar_init(q_full, 1);
+    for (int j = 0; j < kQTiles; ++j) {
+      mbar_init(s_full(j), 1);
+      mbar_init(p_ready(j), 4 * 32);
+    }
+    mbar_init(o_done, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == kLoadWarp) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmQ);
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      mbar_arrive_expect_tx(q_full, kQTiles * C::kQTileBytes);
+      for (int j = 0; j < kQTiles; ++j)
+#pragma unroll
+        for (int p = 0; p < DK / 64; ++p)
+          tma_load_3d(sQ + j * C::kQTileBytes + p * C::kPanelBytes, &tmQ, q_full, p * 64,
+                      q0 + j * kBM, bh);
+      int slot = 0;
+      uint32_t phase = 0;
+      uint32_t issued = 0, issued_phase = 0;  // per slot: a load was issued / its phase bit
+      bool aborted = false;
+      for (int t = 0; t < 2 * n_kt; ++t) {
+        const bool is_k = (t & 1) == 0;
+        const int n = t >> 1;
+        if (!wait_bounded(empty_bar(slot), phase ^ 1u, wc)) {
+          aborted = true;
+          break;
+        }
+        issued |= 1u << slot;
+        issued_phase = (issued_phase & ~(1u << slot)) | (phase << slot);
+        const uint32_t dst = sKV + slot * C::kStageBytes;
+        if (is_k) {
+          mbar_arrive_expect_tx(full_bar(slot), C::kKTileBytes);
+#pragma unroll
+          for (int p = 0; p < DK / 64; ++p)
+            tma_load_3d(dst + p * C::kPanelBytes, &tmK, full_bar(slot), p * 64, n * kBN, bh);
+        } else {
+          mbar_arrive_expect_tx(full_bar(slot), C::kVTileBytes);
+#pragma unroll
+          for (int p = 0; p < DV / 64; ++p)
+            tma_load_3d(dst + p * C::kPanelBytes, &tmV, full_bar(slot), p * 64, n * kBN, bh);
+        }
+        if (++slot == C::kStages) {
+          slot = 0;
+          phase ^= 1u;
+        }
+      }
+      if (aborted || *abort_flag) {
+        // Let every copy already issued land before the CTA can exit.
+        wait_quiesce(q_full, 0, wait_limit_ns);
+        for (int sl = 0; sl < C::kStages; ++sl)
+          if (issued & (1u << sl)) wait_quiesce(full_bar(sl), (issued_phase >> sl) & 1u, wait_limit_ns);
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t kIdescQK = make_idesc(kBM, kBN, false);
+      constexpr uint32_t kIdescPV = make_idesc(kBM, 64, true);
+      const uint32_t tS[2] = {tmem + C::kTmemS0, tmem + C::kTmemS1};
+      const uint32_t tO[2] = {tmem + C::kTmemO0, tmem + C::kTmemO1};
+      int slot = 0;
+      uint32_t phase = 0;
+      auto next = [&]() {
+        if (++slot == C::kStages) {
+          slot = 0;
+          phase ^= 1u;
+        }
+      };
+      // S_j = Q_j K^T over d_k in steps of 16: panel p = kk/4, 32-byte step inside the panel.
+      auto issue_qk = [&](int j, int kslot) {
+        const uint32_t a0 = sQ + j * C::kQTileBytes;
+        const uint32_t b0 = sKV + kslot * C::kStageBytes;
+#pragma unroll
+        for (int kk = 0; kk < DK / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * C::kPanelBytes + (kk & 3) * 32;
+          mma_f16_ss(tS[j], make_sdesc_sw128(a0 + off, 16, 1024),
+                     make_sdesc_sw128(b0 + off, 16, 1024), kIdescQK, kk > 0 ? 1u : 0u);
+        }
+      };
+      // O_j (+)= P_j V: A = P_j from TMEM (bf16 pairs, 8 columns per 16 keys), B = V tile
+      // (MN-major: 16 keys = two 8-row groups 1024 B apart; one 64-column panel per N=64 MMA).
+      auto issue_pv = [&](int j, int vslot, bool accumulate) {
+        const uint32_t b0 = sKV + vslot * C::kStageBytes;
+#pragma unroll
+        for (int kk = 0; kk < kBN / 16; ++kk)
+#pragma unroll
+          for (int h = 0; h < DV / 64; ++h)
+            mma_f16_ts(tO[j] + h * 64, tS[j] + kk * 8,
+                       make_sdesc_sw128(b0 + h * C::kPanelBytes + kk * 2048, 1024, 1024),
+                       kIdescPV, (accumulate || kk > 0) ? 1u : 0u);
+      };
+      bool ok = wait_bounded(q_full, 0, wc);
+      if (ok) ok = wait_bounded(full_bar(slot), phase, wc);
+      if (ok) {
+        tc_fence_after_sync();
+        const int ks = slot;
+        next();
+        for (int j = 0; j < kQTiles; ++j) {
+          issue_qk(j, ks);
+          mma_commit(s_full(j));
+        }
+        mma_commit(empty_bar(ks));
+      }
+      for (int n = 1; ok && n < n_kt; ++n) {
+        const int vs = slot;
+        ok = wait_bounded(full_bar(slot), phase, wc);
+        next();
+        const int ks = slot;
+        if (ok) ok = wait_bounded(full_bar(slot), phase, wc);
+        next();
+        for (int j = 0; ok && j < kQTiles; ++j) {
+          ok = wait_bounded(p_ready(j), uint32_t(n - 1) & 1u, wc);
+          if (!ok) break;
+          tc_fence_after_sync();
+          issue_pv(j, vs, n - 1 > 0);
+          issue_qk(j, ks);
+          mma_commit(s_full(j));
+        }
+        if (ok) {
+          mma_commit(empty_bar(vs));
+          mma_commit(empty_bar(ks));
+        }
+      }
+      if (ok) {
+        const int vs = slot;
+        ok = wait_bounded(full_bar(slot), phase, wc);
+        for (int j = 0; ok && j < kQTiles; ++j) {
+          ok = wait_bounded(p_ready(j), uint32_t(n_kt - 1) & 1u, wc);
+          if (!ok) break;
+          tc_fence_after_sync();
+          issue_pv(j, vs, n_kt - 1 > 0);
+        }
+        if (ok) mma_commit(empty_bar(vs));
+      }
+      // Always signal the epilogue barrier once everything issued has completed, so that the
+      // TMEM is quiescent before it is freed even on the abort path.
+      mma_commit(o_done);
+    }
+  } else {
+    // ---------------------------------------------------------------- softmax warpgroups
+    const int j = warp >> 2;                // Q tile of this warpgroup
+    const int lane_base = (warp & 3) * 32;  // TMEM lanes of this warp
+    const int row = lane_base + lane;       // query row inside the tile
+    const uint32_t tS = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemS1 : C::kTmemS0);
+    const uint32_t tO = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemO1 : C::kTmemO0);
+    const bool neg = c_log2 < 0.f;
+    float m = -INFINITY;  // running maximum of c_log2 * s (log2 units)
+    float l = 0.f;        // running sum of exp2(c_log2 * s - m)
+    bool ok = true;
+    for (int n = 0; n < n_kt; ++n) {
+      if (!wait_bounded(s_full(j), uint32_t(n) & 1u, wc)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after_sync();
+      uint32_t sr[128];
+      tmem_load_row128(tS, sr);
+      float* s = reinterpret_cast<float*>(sr);
+      const int valid = min(kBN, Nk - n * kBN);
+      // Step I: maximum of the scaled scores of this tile (max of s if c >= 0, else min).
+      float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
+      if (valid == kBN) {
+        if (!neg) {
+#pragma unroll
+          for (int i = 0; i < kBN; i += 4) {
+            mx0 = fmaxf(mx0, s[i]);
+            mx1 = fmaxf(mx1, s[i + 1]);
+            mx2 = fmaxf(mx2, s[i + 2]);
+            mx3 = fmaxf(mx3, s[i + 3]);
+          }
+        } else {
+#pragma unroll
+          for (int i = 0; i < kBN; i += 4) {
+            mx0 = fmaxf(mx0, -s[i]);
+            mx1 = fmaxf(mx1, -s[i + 1]);
+            mx2 = fmaxf(mx2, -s[i + 2]);
+            mx3 = fmaxf(mx3, -s[i + 3]);
+          }
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < kBN; ++i)
+          if (i < valid) mx0 = fmaxf(mx0, neg ? -s[i] : s[i]);
+      }
+      const float tmax = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3));
+      const float m_tile = neg ? -c_log2 * tmax : c_log2 * tmax;  // max_k of c_log2 * s_k
+      if (n == 0) {
+        m = m_tile;
+      } else {
+        const bool need = m_tile > m + kRescaleLog2;
+        if (__any_sync(0xffffffffu, need)) {
+          const float m_new = fmaxf(m, m_tile);
+          const float alpha = ex2_approx(m - m_new);
+          l *= alpha;
+          // O_j holds P V of tiles < n (complete: S_j(n) was committed after that product).
+          tmem_scale_row<DV>(tO, alpha);
+          m = m_new;
+        }
+      }
+      // Step II + III: p = exp2(c*s - m), row sum, P -> bf16 pairs into the S columns.
+      const float neg_m = -m;
+      float l0 = 0.f, l1 = 0.f;
+      uint32_t pk[64];
+      if (valid == kBN) {
+#pragma unroll
+        for (int i = 0; i < kBN; i += 2) {
+          const float p0 = ex2_approx(fmaf(s[i], c_log2, neg_m));
+          const float p1 = ex2_approx(fmaf(s[i + 1], c_log2, neg_m));
+          l0 += p0;
+          l1 += p1;
+          pk[i >> 1] = pack_bf16x2(p0, p1);
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < kBN; i += 2) {
+          const float p0 = (i < valid) ? ex2_approx(fmaf(s[i], c_log2, neg_m)) : 0.f;
+          const float p1 = (i + 1 < valid) ? ex2_approx(fmaf(s[i + 1], c_log2, neg_m)) : 0.f;
+          l0 += p0;
+          l1 += p1;
+          pk[i >> 1] = pack_bf16x2(p0, p1);
+        }
+      }
+      l += l0 + l1;
+      tmem_st_32x32b_x32(tS + 0, pk);
+      tmem_st_32x32b_x32(tS + 32, pk + 32);
+      tmem_wait_st();
+      tc_fence_before_sync();
+      mbar_arrive(p_ready(j));
+    }
+    // Epilogue, Step IV: O / l -> bf16 -> global.
+    if (ok && wait_bounded(o_done, 0, wc)) {
+      tc_fence_after_sync();
+      const float inv_l = 1.0f / l;
+      const int grow = q0 + j * kBM + row;
+      __nv_bfloat16* orow = O + (size_t(bh) * Nq + grow) * DV;
+#pragma unroll
+      for (int c = 0; c < DV; c += 32) {
+        uint32_t o[32];
+        tmem_ld_32x32b_x32(tO + c, o);
+        tmem_wait_ld();
+        reg_anchor_x32(o);
+        if (grow < Nq) {
+          uint4 pkt[4];
+          uint32_t* w = reinterpret_cast<uint32_t*>(pkt);
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            w[i] = pack_bf16x2(__uint_as_float(o[2 * i]) * inv_l,
+                               __uint_as_float(o[2 * i + 1]) * inv_l);
+          uint4* dst = reinterpret_cast<uint4*>(orow + c);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) dst[i] = pkt[i];
+        }
+      }
+    }
+  }
+
+  // Teardown: wait for the tensor core to go quiet before freeing TMEM.
+  if (warp == kMmaWarp) wait_quiesce(o_done, 0, wait_limit_ns);
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after_sync();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// Host side
+// ------------------------------------------------------------------------------------------
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn(char* msg, size_t msglen) {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  static char err[256] = {0};
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                                     cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || p == nullptr) {
+      snprintf(err, sizeof(err), "cuTensorMapEncodeTiled unavailable: %s",
+               cudaGetErrorString(e));
+      return;
+    }
+    fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  if (!fn) snprintf(msg, msglen, "%s", err);
+  return fn;
+}
+
+// 3-D map over a contiguous [BH, N, d] bf16 tensor; box = 64 columns x 128 rows x 1 slice,
+// 128-byte swizzle.  Rows past N inside a slice read as zero (never the next slice).
+bool encode_map(EncodeTiledFn enc, CUtensorMap* map, const void* base, int64_t BH, int64_t N,
+                int64_t d, char* msg, size_t msglen) {
+  const cuuint64_t dims[3] = {cuuint64_t(d), cuuint64_t(N), cuuint64_t(BH)};
+  const cuuint64_t strides[2] = {cuuint64_t(d * 2), cuuint64_t(N * d * 2)};
+  const cuuint32_t box[3] = {64, 128, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims,
+                   strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    snprintf(msg, msglen, "cuTensorMapEncodeTiled failed (%d) for [%lld,%lld,%lld]", int(r),
+             (long long)BH, (long long)N, (long long)d);
+    return false;
+  }
+  return true;
+}
+
+template <int DK, int DV>
+int launch_tc(const AttnArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
+              const CUtensorMap& mv, char* msg, size_t msglen) {
+  using C = Cfg<DK, DV>;
+  auto kern = attn_fwd_bf16_tc_kernel<DK, DV>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [&] {
+    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    C::kSmemBytes);
+  });
+  if (attr_err != cudaSuccess) {
+    snprintf(msg, msglen, "cudaFuncSetAttribute (bf16 kernel): %s", cudaGetErrorString(attr_err));
+    return 5;
+  }
+  const int64_t n_qblocks = (a.Nq + kQTiles * kBM - 1) / (kQTiles * kBM);
+  const int64_t grid = a.B * a.H * n_qblocks;
+  if (grid > 0x7fffffffLL) {
+    snprintf(msg, msglen, "bf16 path: %lld CTAs exceeds the grid limit", (long long)grid);
+    return 3;
+  }
+  const float c_log2 = a.scale * 1.4426950408889634f;
+  kern<<<dim3(unsigned(grid)), dim3(kThreads), C::kSmemBytes, a.stream>>>(
+      mq, mk, mv, static_cast<__nv_bfloat16*>(a.O), int(a.Nq), int(a.Nk), int(n_qblocks), c_log2,
+      wait_limit_ns());
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    snprintf(msg, msglen, "bf16 kernel launch: %s", cudaGetErrorString(e));
+    return 5;
+  }
+  return 0;
+}
+
+}  // namespace
+
+int launch_attn_fwd_bf16(const AttnArgs& a, char* msg, size_t msglen) {
+  EncodeTiledFn enc = get_encode_fn(msg, msglen);
+  if (!enc) return 5;
+  const int64_t BH = a.B * a.H;
+  CUtensorMap mq, mk, mv;
+  if (!encode_map(enc, &mq, a.Q, BH, a.Nq, a.dk, msg, msglen)) return 5;
+  if (!encode_map(enc, &mk, a.K, BH, a.Nk, a.dk, msg, msglen)) return 5;
+  if (!encode_map(enc, &mv, a.V, BH, a.Nk, a.dv, msg, msglen)) return 5;
+  if (a.dk == 64 && a.dv == 64) return launch_tc<64, 64>(a, mq, mk, mv, msg, msglen);
+  if (a.dk == 128 && a.dv == 128) return launch_tc<128, 128>(a, mq, mk, mv, msg, msglen);
+  if (a.dk == 128 && a.dv == 64) return launch_tc<128, 64>(a, mq, mk, mv, msg, msglen);
+  if (a.dk == 64 && a.dv == 128) return launch_tc<64, 128>(a, mq, mk, mv, msg, msglen);
+  snprintf(msg, msglen, "bf16 path supports d_k, d_v in {64, 128}; got d_k=%lld d_v=%lld",
+           (long long)a.dk, (long long)a.dv);
+  return 3;
+}
+
+cudaError_t bf16_read_and_clear_status(unsigned* value) {
+  cudaError_t e = cudaMemcpyFromSymbol(value, g_moa_bf16_status, sizeof(unsigned));
+  if (e != cudaSuccess) return e;
+  const unsigned zero = 0;
+  return cudaMemcpyToSymbol(g_moa_bf16_status, &zero, sizeof(unsigned));
+}
+
+}  // namespace moa

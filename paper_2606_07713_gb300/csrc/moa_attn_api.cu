@@ -1,0 +1,185 @@
+// C ABI of libmoa_attn.so: argument checks, dispatch to the kernels, status and helpers.
+// The contract of every entry point is documented in include/moa_attn.h.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdint>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+
+#include "../../include/moa_attn.h"
+#include "internal.h"
+
+namespace moa {
+
+uint64_t wait_limit_ns() {
+  static const uint64_t v = [] {
+    const char* s = std::getenv("MOA_WAIT_LIMIT_NS");
+    if (s && *s) {
+      const unsigned long long x = std::strtoull(s, nullptr, 10);
+      if (x > 0) return uint64_t(x);
+    }
+    return uint64_t(1000000000ull);  // 1 s
+  }();
+  return v;
+}
+
+namespace {
+
+thread_local char t_last_error[512] = {0};
+
+int fail(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(t_last_error, sizeof(t_last_error), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+// a * b for non-negative values, or -1 on overflow of int64.
+int64_t mul_checked(int64_t a, int64_t b) {
+  if (a < 0 || b < 0) return -1;
+  if (a != 0 && b > INT64_MAX / a) return -1;
+  return a * b;
+}
+
+int64_t numel4(int64_t a, int64_t b, int64_t c, int64_t d) {
+  int64_t x = mul_checked(a, b);
+  x = x < 0 ? -1 : mul_checked(x, c);
+  return x < 0 ? -1 : mul_checked(x, d);
+}
+
+bool overlaps(const void* a, int64_t abytes, const void* b, int64_t bbytes) {
+  const uintptr_t a0 = reinterpret_cast<uintptr_t>(a), b0 = reinterpret_cast<uintptr_t>(b);
+  return a0 < b0 + uintptr_t(bbytes) && b0 < a0 + uintptr_t(abytes);
+}
+
+// Checks everything that can be checked without touching the device.  On success fills *sz
+// with the byte sizes of Q, K, V, O.
+int validate(const void* Q, const void* K, const void* V, void* O, int64_t B, int64_t H,
+             int64_t Nq, int64_t Nk, int64_t dk, int64_t dv, float scale, int dtype,
+             int64_t sz[4]) {
+  if (!Q || !K || !V || !O) return fail(MOA_ERR_INVALID_ARG, "null tensor pointer");
+  if (B <= 0 || H <= 0 || Nq <= 0 || Nk <= 0 || dk <= 0 || dv <= 0)
+    return fail(MOA_ERR_INVALID_ARG,
+                "sizes must be >= 1 (B=%lld H=%lld N_q=%lld N_k=%lld d_k=%lld d_v=%lld)",
+                (long long)B, (long long)H, (long long)Nq, (long long)Nk, (long long)dk,
+                (long long)dv);
+  if (!std::isfinite(scale)) return fail(MOA_ERR_INVALID_ARG, "scale must be finite");
+  if (dtype != MOA_FP32 && dtype != MOA_BF16)
+    return fail(MOA_ERR_UNSUPPORTED_DTYPE, "unknown dtype %d", dtype);
+  const int64_t elt = dtype == MOA_FP32 ? 4 : 2;
+  const int64_t nq = numel4(B, H, Nq, dk), nk = numel4(B, H, Nk, dk);
+  const int64_t nv = numel4(B, H, Nk, dv), no = numel4(B, H, Nq, dv);
+  if (nq < 0 || nk < 0 || nv < 0 || no < 0 || nq > INT64_MAX / 4 || nk > INT64_MAX / 4 ||
+      nv > INT64_MAX / 4 || no > INT64_MAX / 4)
+    return fail(MOA_ERR_UNSUPPORTED_SHAPE, "tensor sizes overflow 64-bit byte counts");
+  if (B * H > 0x7fffffffLL || Nq > 0x7fffffffLL || Nk > 0x7fffffffLL)
+    return fail(MOA_ERR_UNSUPPORTED_SHAPE, "B*H, N_q and N_k must each be below 2^31");
+  if (dtype == MOA_BF16) {
+    if ((dk != 64 && dk != 128) || (dv != 64 && dv != 128))
+      return fail(MOA_ERR_UNSUPPORTED_SHAPE, "bf16 needs d_k, d_v in {64, 128}; got %lld, %lld",
+                  (long long)dk, (long long)dv);
+  } else {
+    if (dk > 128 || dv > 128)
+      return fail(MOA_ERR_UNSUPPORTED_SHAPE, "fp32 needs d_k, d_v <= 128; got %lld, %lld",
+                  (long long)dk, (long long)dv);
+    if (dk % 4 != 0 || dv % 4 != 0)
+      return fail(MOA_ERR_MISALIGNED, "fp32 rows must be multiples of 16 bytes (d %% 4 == 0)");
+  }
+  const void* ptrs[4] = {Q, K, V, O};
+  for (const void* p : ptrs)
+    if (reinterpret_cast<uintptr_t>(p) % 16 != 0)
+      return fail(MOA_ERR_MISALIGNED, "tensor pointer %p is not 16-byte aligned", p);
+  sz[0] = nq * elt;
+  sz[1] = nk * elt;
+  sz[2] = nv * elt;
+  sz[3] = no * elt;
+  if (overlaps(O, sz[3], Q, sz[0]) || overlaps(O, sz[3], K, sz[1]) ||
+      overlaps(O, sz[3], V, sz[2]))
+    return fail(MOA_ERR_INVALID_ARG, "O overlaps an input tensor");
+  return MOA_OK;
+}
+
+int dispatch(const void* Q, const void* K, const void* V, void* O, int64_t B, int64_t H,
+             int64_t Nq, int64_t Nk, int64_t dk, int64_t dv, float scale, int dtype,
+             void* stream) {
+  AttnArgs a{Q, K, V, O, B, H, Nq, Nk, dk, dv, scale, static_cast<cudaStream_t>(stream)};
+  char msg[256] = {0};
+  const int rc = dtype == MOA_BF16 ? launch_attn_fwd_bf16(a, msg, sizeof(msg))
+                                   : launch_attn_fwd_f32(a, msg, sizeof(msg));
+  if (rc != MOA_OK) return fail(rc, "%s", msg);
+  t_last_error[0] = '\0';
+  return MOA_OK;
+}
+
+}  // namespace
+}  // namespace moa
+
+extern "C" {
+
+int moa_attn_fwd(const void* Q, const void* K, const void* V, void* O, int64_t B, int64_t H,
+                 int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v, float scale, int dtype,
+                 void* stream) {
+  int64_t sz[4];
+  const int rc = moa::validate(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
+  if (rc != MOA_OK) return rc;
+  return moa::dispatch(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream);
+}
+
+int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO, void* dQ,
+                        void* dK, void* dV, void* dO, int64_t B, int64_t H, int64_t N_q,
+                        int64_t N_k, int64_t d_k, int64_t d_v, float scale, int dtype,
+                        void* stream) {
+  if (!hQ || !hK || !hV || !hO) return moa::fail(MOA_ERR_INVALID_ARG, "null host pointer");
+  int64_t sz[4];
+  int rc = moa::validate(dQ, dK, dV, dO, B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
+  if (rc != MOA_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const void* src[3] = {hQ, hK, hV};
+  void* dst[3] = {dQ, dK, dV};
+  for (int i = 0; i < 3; ++i) {
+    cudaError_t e = cudaMemcpyAsync(dst[i], src[i], size_t(sz[i]), cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess)
+      return moa::fail(MOA_ERR_CUDA, "host-to-device copy: %s", cudaGetErrorString(e));
+  }
+  rc = moa::dispatch(dQ, dK, dV, dO, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream);
+  if (rc != MOA_OK) return rc;
+  cudaError_t e = cudaMemcpyAsync(hO, dO, size_t(sz[3]), cudaMemcpyDeviceToHost, s);
+  if (e != cudaSuccess)
+    return moa::fail(MOA_ERR_CUDA, "device-to-host copy: %s", cudaGetErrorString(e));
+  return MOA_OK;
+}
+
+const char* moa_last_error(void) { return moa::t_last_error; }
+
+int moa_get_device_status(void* stream) {
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess)
+    return moa::fail(MOA_ERR_CUDA, "stream synchronize: %s", cudaGetErrorString(e));
+  unsigned v = 0;
+  e = moa::bf16_read_and_clear_status(&v);
+  if (e != cudaSuccess)
+    return moa::fail(MOA_ERR_CUDA, "status word read: %s", cudaGetErrorString(e));
+  if (v != 0)
+    return moa::fail(MOA_ERR_DEVICE_TIMEOUT, "a kernel wait ran out (status %u)", v);
+  return MOA_OK;
+}
+
+double moa_attn_flops(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v) {
+  return 2.0 * double(B) * double(H) * double(N_q) * double(N_k) * double(d_k + d_v);
+}
+
+double moa_attn_dnf_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int64_t d_k,
+                          int64_t d_v, int dtype) {
+  const double elt = dtype == MOA_FP32 ? 4.0 : dtype == MOA_BF16 ? 2.0 : -1.0;
+  if (elt < 0) return -1.0;
+  return elt * double(B) * double(H) *
+         (double(N_q) * d_k + double(N_k) * d_k + double(N_k) * d_v + double(N_q) * d_v);
+}
+
+int moa_attn_version(void) { return 100; }
+
+}  // extern "C"

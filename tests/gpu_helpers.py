@@ -1,0 +1,37 @@
+"""Helpers for the GPU tests: move generated inputs to the device and compare with the oracle."""
+from __future__ import annotations
+
+import numpy as np
+
+BF16_TOL = 2e-2   # max|O - O_ref| <= BF16_TOL * max|O_ref| (bf16 inputs, fp32 accumulation)
+FP32_TOL = 1e-5   # same bound for fp32 inputs
+
+
+def to_device(x, dev="cuda:0"):
+    """AttnInputs -> (q, k, v) torch tensors on dev in the workload's storage type."""
+    import torch
+    if x.cfg.dtype == "bf16":
+        conv = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+        return conv(x.q_bits), conv(x.k_bits), conv(x.v_bits)
+    return tuple(torch.from_numpy(np.ascontiguousarray(a)).to(dev) for a in (x.q, x.k, x.v))
+
+
+def bf16_tensor_from_f32(a, dev="cuda:0"):
+    """Exact bf16 tensor from float32 values that are already bf16-representable."""
+    import torch
+    from paper_2606_07713_gb300 import inputs as I
+    bits = I.f32_to_bf16_bits(np.asarray(a, dtype=np.float32))
+    assert np.array_equal(I.bf16_bits_to_f32(bits), np.asarray(a, dtype=np.float32))
+    return torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).to(dev)
+
+
+def rel_err(o_gpu: np.ndarray, o_ref: np.ndarray) -> float:
+    return float(np.max(np.abs(o_gpu.astype(np.float64) - o_ref)) / np.max(np.abs(o_ref)))
+
+
+def assert_close(o_gpu, o_ref, dtype: str, what: str = ""):
+    tol = BF16_TOL if dtype == "bf16" else FP32_TOL
+    err = rel_err(o_gpu, o_ref)
+    assert np.all(np.isfinite(o_gpu)), f"{what}: non-finite output"
+    assert err <= tol, f"{what}: max|O-O_ref|/max|O_ref| = {err:.3e} > {tol}"
+    return err

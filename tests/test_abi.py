@@ -1,0 +1,91 @@
+"""The C ABI without a GPU: the library loads, exports every declared symbol, and rejects bad
+arguments with the documented status codes before launching anything."""
+import math
+import os
+import re
+
+import pytest
+
+import paper_2606_07713_gb300 as pkg
+from paper_2606_07713_gb300 import _lib
+from paper_2606_07713_gb300 import inputs as I
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "moa_attn.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2606_07713_gb300 import build
+    build.build()
+    return _lib.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(moa_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    assert "moa_attn_fwd" in names and "moa_get_device_status" in names
+    assert set(names) == set(_lib.SIGNATURES), "binding and header disagree"
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+    assert pkg.moa_attn_version() >= 100
+
+
+def test_flops_and_dnf_bytes_helpers(L):
+    for cid, cfg in I.CONFIGS.items():
+        s = cfg.shape
+        f = pkg.attn_flops(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v)
+        assert f == 2.0 * s.B * s.H * s.N_q * s.N_k * (s.d_k + s.d_v)
+        elt = 4 if cfg.dtype == "fp32" else 2
+        code = pkg.MOA_FP32 if cfg.dtype == "fp32" else pkg.MOA_BF16
+        b = pkg.dnf_bytes(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v, code)
+        assert b == elt * (s.numel_q + s.numel_k + s.numel_v + s.numel_o)
+    assert math.isclose(pkg.attn_flops(2, 32, 8192, 8192, 128, 128), 2.199023e12, rel_tol=1e-6)
+    assert pkg.dnf_bytes(1, 1, 1, 1, 1, 1, 9) == -1.0
+
+
+# Fake, never dereferenced device addresses: validation fails before any CUDA call.
+A, B_, C, D = 0x100000, 0x200000, 0x300000, 0x400000
+
+
+def call(Q=A, K=B_, V=C, O=D, B=1, H=1, Nq=8, Nk=8, dk=64, dv=64, scale=0.125, dtype=1):
+    return _lib.moa_attn_fwd(Q, K, V, O, B, H, Nq, Nk, dk, dv, scale, dtype, None)
+
+
+@pytest.mark.parametrize("kwargs,code", [
+    (dict(Q=None), _lib.MOA_ERR_INVALID_ARG),
+    (dict(O=None), _lib.MOA_ERR_INVALID_ARG),
+    (dict(B=0), _lib.MOA_ERR_INVALID_ARG),
+    (dict(Nk=0), _lib.MOA_ERR_INVALID_ARG),
+    (dict(dv=-1), _lib.MOA_ERR_INVALID_ARG),
+    (dict(scale=float("nan")), _lib.MOA_ERR_INVALID_ARG),
+    (dict(scale=float("inf")), _lib.MOA_ERR_INVALID_ARG),
+    (dict(dtype=7), _lib.MOA_ERR_UNSUPPORTED_DTYPE),
+    (dict(dk=96), _lib.MOA_ERR_UNSUPPORTED_SHAPE),
+    (dict(dv=256), _lib.MOA_ERR_UNSUPPORTED_SHAPE),
+    (dict(dtype=0, dk=132), _lib.MOA_ERR_UNSUPPORTED_SHAPE),
+    (dict(dtype=0, dv=6), _lib.MOA_ERR_MISALIGNED),
+    (dict(Q=A + 8), _lib.MOA_ERR_MISALIGNED),
+    (dict(O=D + 2), _lib.MOA_ERR_MISALIGNED),
+    (dict(O=A), _lib.MOA_ERR_INVALID_ARG),              # O aliases Q
+    (dict(O=C + 16), _lib.MOA_ERR_INVALID_ARG),         # O overlaps V
+    (dict(Nq=2 ** 31), _lib.MOA_ERR_UNSUPPORTED_SHAPE),
+    (dict(B=2 ** 20, H=2 ** 12), _lib.MOA_ERR_UNSUPPORTED_SHAPE),
+    (dict(B=2 ** 40, Nq=2 ** 20), _lib.MOA_ERR_UNSUPPORTED_SHAPE),
+])
+def test_validation_rejects_before_launch(L, kwargs, code):
+    assert call(**kwargs) == code
+    assert _lib.moa_last_error() != ""
+
+
+def test_staged_rejects_null_host_pointers(L):
+    rc = _lib.moa_attn_fwd_staged(None, A, A, A, A, B_, C, D, 1, 1, 8, 8, 64, 64, 0.1, 1, None)
+    assert rc == _lib.MOA_ERR_INVALID_ARG
