@@ -1,0 +1,386 @@
+"""Benchmark of the DNF attention forward on GB300.
+
+Default workload: bf16 SDPA forward, B=4, H=16, N_q=N_k=2048, d_k=d_v=64, Q/K/V i.i.d.
+N(0,1) from the seeded generator, scale=1/sqrt(d_k), no mask.  One step = one attention
+forward over that batch (the whole hot path: one kernel launch).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload ID]
+
+Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s: FLOPs of every step on every
+rank divided by the slowest rank's summed kernel time, measured with CUDA events on the
+launching stream, with L2 flushed (a 256 MiB write) before every step.  `e2e` is the same
+metric through moa_attn_fwd_staged (host buffers in and out, copies inside the timed region).
+`--impl reference` times the fp64 CPU oracle on the host cores instead (a bounded sample of
+rows per step).  Multi-GPU (torchrun): every rank runs its own full copy of the workload (the
+(b, h) problems are independent; no collective on the data path), so scaling is weak.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2606_07713_gb300 import inputs as I  # noqa: E402
+
+METRIC = "attention fwd TFLOP/s and % of GB300 bf16 peak; DRAM bytes vs DNF minimum"
+DEFAULT_WORKLOAD = 2
+PROFILE = os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b4h16n2048d64.txt")
+KERNEL_SOURCES = [os.path.join(ROOT, "paper_2606_07713_gb300", "csrc", f)
+                  for f in ("attn_fwd_bf16_tc.cu", "ptx.cuh")]
+FLUSH_BYTES = 256 << 20
+
+
+def workload_desc(cfg: I.AttnConfig) -> dict:
+    s = cfg.shape
+    v = "U[-1,1]" if cfg.v_dist == "uniform" else "N(0,1)"
+    desc = (f"{cfg.dtype} SDPA fwd, B={s.B}, H={s.H}, N_q={s.N_q}, N_k={s.N_k}, d_k={s.d_k}, "
+            f"d_v={s.d_v}, Q~{cfg.q_sigma:g}*N(0,1), K~{cfg.k_sigma:g}*N(0,1), V~{v}, "
+            f"scale=1/sqrt(d_k), no mask")
+    if cfg.plants_per_head:
+        desc += f", {cfg.plants_per_head} planted one-hot rows per head"
+    return {"workload": desc, "B": s.B, "H": s.H, "N_q": s.N_q, "N_k": s.N_k, "d_k": s.d_k,
+            "d_v": s.d_v, "seed": cfg.the_seed,
+            "l2": f"flushed before every step ({FLUSH_BYTES >> 20} MiB write, untimed)"}
+
+
+def measured_peaks() -> tuple[dict, str]:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        return json.load(open(p)), "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        h.update(open(f, "rb").read())
+    return h.hexdigest()
+
+
+def profiled_traffic() -> tuple[float | None, float | None]:
+    """(DRAM bytes per launch, ncu duration) from the committed ncu summary, if it was captured
+    from the current kernel source; (None, None) otherwise."""
+    try:
+        text = open(PROFILE).read()
+    except OSError:
+        return None, None
+    m = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", text)
+    b = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    if not m or not b or m.group(1) != kernel_source_hash():
+        return None, None
+    return float(b.group(1)), None
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle sampling while the timed loop runs."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines: list[str] = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons, power = [], [], set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+                power.append(float(f[3]))
+            except ValueError:
+                continue
+            for n, val in zip(names, f[5:9]):
+                if val.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(smax), "samples": len(sm),
+                "power_w_max": max(power) if power else None, "reasons": sorted(reasons)}
+
+
+def to_device_bf16(bits, dev):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+
+
+# ------------------------------------------------------------------------------------------
+# our arm
+# ------------------------------------------------------------------------------------------
+def run_ours(args, cfg: I.AttnConfig) -> None:
+    import torch
+    import torch.distributed as dist
+
+    import paper_2606_07713_gb300 as pkg
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    pkg.lib()
+    s = cfg.shape
+    x = I.make_inputs(cfg)
+    if cfg.dtype == "bf16":
+        q, k, v = (to_device_bf16(b, dev) for b in (x.q_bits, x.k_bits, x.v_bits))
+        hq, hk, hv = (torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).view(torch.bfloat16)
+                      .pin_memory() for b in (x.q_bits, x.k_bits, x.v_bits))
+    else:
+        q, k, v = (torch.from_numpy(a).to(dev) for a in (x.q, x.k, x.v))
+        hq, hk, hv = (torch.from_numpy(a).pin_memory() for a in (x.q, x.k, x.v))
+    o = torch.empty((s.B, s.H, s.N_q, s.d_v), dtype=q.dtype, device=dev)
+    ho = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flops = pkg.attn_flops(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v)
+    code = pkg.MOA_BF16 if cfg.dtype == "bf16" else pkg.MOA_FP32
+    dnf = pkg.dnf_bytes(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v, code)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        pkg.attn_fwd(q, k, v, cfg.scale, out=o)
+    torch.cuda.synchronize(dev)
+    pkg.check(pkg.get_device_status())
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    barrier()
+    t_wall = time.perf_counter()
+    for i in range(args.steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        pkg.attn_fwd(q, k, v, cfg.scale, out=o, stream=stream)
+        ev[i][1].record(stream)
+    barrier()
+    wall = time.perf_counter() - t_wall
+    kern_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = float(np.sum(kern_ms))
+
+    # end to end: host buffers in, result back to the host, through the C ABI
+    ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    barrier()
+    for i in range(args.steps):
+        flush.zero_()
+        ev2[i][0].record(stream)
+        pkg.attn_fwd_staged(hq, hk, hv, ho, q, k, v, o, cfg.scale, stream=stream)
+        ev2[i][1].record(stream)
+    barrier()
+    clocks = sampler.stop()
+    e2e_ms = float(np.sum([a.elapsed_time(b) for a, b in ev2]))
+    pkg.check(pkg.get_device_status())
+
+    if world > 1:
+        t = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms, e2e_ms = float(t[0]), float(t[1])
+
+    if rank == 0:
+        peaks, peak_src = measured_peaks()
+        value = flops * args.steps * world / (total_ms * 1e-3) / 1e12
+        per_launch_ms = float(np.mean(kern_ms))
+        achieved = flops / (per_launch_ms * 1e-3) / 1e12
+        peak = float(peaks["bf16_tflops"]) if cfg.dtype == "bf16" else None
+        traffic, _ = profiled_traffic()
+        line = {
+            "metric": METRIC,
+            "value": round(value, 2),
+            "unit": "TFLOP/s",
+            "n_gpus": world,
+            "steps": args.steps,
+            "warmup": args.warmup,
+            "ms_per_step": round(total_ms / args.steps, 6),
+            "higher_is_better": True,
+            "scaling": "weak",
+            "vs_baseline": None,
+            "dtype": cfg.dtype,
+            "data": "synthetic: seeded splitmix64 + Box-Muller inputs of the workload's shape",
+            "config": workload_desc(cfg),
+            "pct_of_bf16_peak": round(100.0 * achieved / float(peaks["bf16_tflops"]), 2),
+            "dnf_bytes": dnf,
+            "roofline": {
+                "bound": "tensor",
+                "achieved": round(achieved, 2),
+                "peak": peak,
+                "peak_source": f"{peak_src} bf16_tflops (burst; kernel timed alone)",
+                "unit": "TFLOP/s",
+                "frac": round(achieved / peak, 4) if peak else None,
+                "traffic": traffic,
+                "traffic_vs_dnf": round(traffic / dnf, 4) if traffic else None,
+                "kernel": "attn_fwd_bf16_tc_kernel" if cfg.dtype == "bf16" else "attn_fwd_f32_cc_kernel",
+            },
+            "e2e": {
+                "value": round(flops * args.steps * world / (e2e_ms * 1e-3) / 1e12, 2),
+                "unit": "TFLOP/s",
+                "h2d_bytes_per_step": int(hq.numel() * hq.element_size() + hk.numel() * hk.element_size()
+                                          + hv.numel() * hv.element_size()),
+                "d2h_bytes_per_step": int(ho.numel() * ho.element_size()),
+                "api": "moa_attn_fwd_staged",
+            },
+            "gpu_launches": args.steps,
+            "clocks": clocks,
+            "wall_s_timed_loop": round(wall, 4),
+        }
+        if world == 1:
+            line["cpu_baseline"] = cpu_baseline(cfg, x, budget_s=args.cpu_budget)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+# ------------------------------------------------------------------------------------------
+# the oracle on the host cores (cpu_baseline leg and --impl reference)
+# ------------------------------------------------------------------------------------------
+def _oracle_rows(cfg, x, nrows, seed):
+    s = cfg.shape
+    total = s.B * s.H * s.N_q
+    rng = np.random.default_rng(seed)
+    if nrows >= total:
+        return np.arange(total, dtype=np.int64)
+    return np.sort(rng.choice(total, size=nrows, replace=False)).astype(np.int64)
+
+
+def _cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(cfg, x, budget_s: float = 12.0) -> dict:
+    import oracle
+    orc = oracle.get()
+    s = cfg.shape
+    flops_row = 2.0 * s.N_k * (s.d_k + s.d_v)
+    total = s.B * s.H * s.N_q
+    probe = _oracle_rows(cfg, x, min(total, 256), 1)
+    t0 = time.perf_counter()
+    orc.rows(x.q, x.k, x.v, cfg.scale, probe)
+    dt = time.perf_counter() - t0
+    n = int(min(total, max(256, len(probe) * budget_s / max(dt, 1e-6))))
+    rows = _oracle_rows(cfg, x, n, 2)
+    t0 = time.perf_counter()
+    orc.rows(x.q, x.k, x.v, cfg.scale, rows)
+    dt = time.perf_counter() - t0
+    return {"value": round(flops_row * len(rows) / dt / 1e12, 6), "unit": "TFLOP/s",
+            "cores": orc.max_threads(), "kind": "oracle",
+            "sample": f"{len(rows)} of {total} output rows (seeded, uniform), fp64, {dt:.1f} s"}
+
+
+def run_reference(args, cfg: I.AttnConfig) -> None:
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle
+    orc = oracle.get()
+    x = I.make_inputs(cfg)
+    s = cfg.shape
+    total = s.B * s.H * s.N_q
+    flops_row = 2.0 * s.N_k * (s.d_k + s.d_v)
+    # size each step's sample so the whole run stays within ~2 minutes of CPU time
+    probe = _oracle_rows(cfg, x, min(total, 128), 1)
+    t0 = time.perf_counter()
+    orc.rows(x.q, x.k, x.v, cfg.scale, probe)
+    per_row = (time.perf_counter() - t0) / len(probe)
+    per_step = max(1, min(total, int(120.0 / max(1, args.steps + args.warmup) / max(per_row, 1e-9))))
+    for i in range(args.warmup):
+        orc.rows(x.q, x.k, x.v, cfg.scale, _oracle_rows(cfg, x, per_step, 100 + i))
+    t = 0.0
+    for i in range(args.steps):
+        rows = _oracle_rows(cfg, x, per_step, 1000 + i)
+        t0 = time.perf_counter()
+        orc.rows(x.q, x.k, x.v, cfg.scale, rows)
+        t += time.perf_counter() - t0
+    value = flops_row * per_step * args.steps / t / 1e12
+    sample = f"{per_step} of {total} output rows per step (seeded, uniform), fp64"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s",
+        "n_gpus": int(os.environ.get("WORLD_SIZE", "1")), "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(1e3 * t / args.steps, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic: seeded splitmix64 + Box-Muller inputs of the workload's shape",
+        "config": workload_desc(cfg),
+        "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "cores": orc.max_threads(),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", type=int, default=DEFAULT_WORKLOAD, choices=sorted(I.CONFIGS))
+    ap.add_argument("--cpu-budget", type=float, default=12.0,
+                    help="seconds of oracle time for the cpu_baseline sample")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    cfg = I.CONFIGS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, cfg)
+    else:
+        run_ours(args, cfg)
+
+
+if __name__ == "__main__":
+    main()
