@@ -147,6 +147,49 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Packed fp32 pairs (Blackwell f32x2 ALU forms): one instruction for two lanes of data.
+__device__ __forceinline__ uint64_t pack_f32x2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+// (d0, d1) = (a0, a1) * b + c, with b and c packed pairs.
+__device__ __forceinline__ void ffma2(float& d0, float& d1, float a0, float a1, uint64_t b,
+                                      uint64_t c) {
+  asm("{\n\t.reg .b64 ra, rd;\n\tmov.b64 ra, {%2, %3};\n\t"
+      "fma.rn.f32x2 rd, ra, %4, %5;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "l"(b), "l"(c));
+}
+// (a0, a1) += (b0, b1).
+__device__ __forceinline__ void fadd2(float& a0, float& a1, float b0, float b1) {
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\tmov.b64 ra, {%0, %1};\n\tmov.b64 rb, {%2, %3};\n\t"
+      "add.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "+f"(a0), "+f"(a1)
+      : "f"(b0), "f"(b1));
+}
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+// Maximum of 128 values (of their negations if NEG) with four independent 3-input chains.
+template <bool NEG>
+__device__ __forceinline__ float row_max128(const float* s) {
+  auto v = [&](int i) { return NEG ? -s[i] : s[i]; };
+  float a0 = v(0), a1 = v(1), a2 = v(2), a3 = v(3);
+#pragma unroll
+  for (int i = 4; i < 124; i += 8) {
+    a0 = max3f(a0, v(i), v(i + 1));
+    a1 = max3f(a1, v(i + 2), v(i + 3));
+    a2 = max3f(a2, v(i + 4), v(i + 5));
+    a3 = max3f(a3, v(i + 6), v(i + 7));
+  }
+  a0 = max3f(a0, v(124), v(125));
+  a1 = max3f(a1, v(126), v(127));
+  return max3f(a0, a1, fmaxf(a2, a3));
+}
+
 // Loads 128 fp32 columns of this thread's TMEM lane into s[] and waits for completion.
 __device__ __forceinline__ void tmem_load_row128(uint32_t taddr, uint32_t* s) {
   tmem_ld_32x32b_x32(taddr + 0, s + 0);
@@ -279,11 +322,14 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
   } else if (warp == kMmaWarp) {
     // ---------------------------------------------------------------- MMA issuer
+    // Straight-line issue code: every operand of every tcgen05.mma is a loop invariant or an
+    // unrolled constant offset, so one thread keeps the tensor pipe fed.
     if (lane == 0) {
       constexpr uint32_t kIdescQK = make_idesc(kBM, kBN, false);
-      constexpr uint32_t kIdescPV = make_idesc(kBM, 64, true);
-      const uint32_t tS[2] = {tmem + C::kTmemS0, tmem + C::kTmemS1};
-      const uint32_t tO[2] = {tmem + C::kTmemO0, tmem + C::kTmemO1};
+      constexpr uint32_t kIdescPV = make_idesc(kBM, DV, true);
+      const uint32_t tS0 = tmem + C::kTmemS0, tS1 = tmem + C::kTmemS1;
+      const uint32_t tO0 = tmem + C::kTmemO0, tO1 = tmem + C::kTmemO1;
+      const uint32_t sQ0 = sQ, sQ1 = sQ + C::kQTileBytes;
       int slot = 0;
       uint32_t phase = 0;
       auto next = [&]() {
@@ -292,39 +338,35 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           phase ^= 1u;
         }
       };
-      // S_j = Q_j K^T over d_k in steps of 16: panel p = kk/4, 32-byte step inside the panel.
-      auto issue_qk = [&](int j, int kslot) {
-        const uint32_t a0 = sQ + j * C::kQTileBytes;
-        const uint32_t b0 = sKV + kslot * C::kStageBytes;
+      // S = Q K^T: DK/16 MMAs (M=128, N=128, K=16), both operands K-major; the k-th step is
+      // panel k/4 of the 128-byte-swizzled tile, 32 bytes further for each step inside it.
+      auto issue_qk = [&](uint32_t tS, uint32_t qa, uint32_t kb) {
 #pragma unroll
         for (int kk = 0; kk < DK / 16; ++kk) {
           const uint32_t off = (kk >> 2) * C::kPanelBytes + (kk & 3) * 32;
-          mma_f16_ss(tS[j], make_sdesc_sw128(a0 + off, 16, 1024),
-                     make_sdesc_sw128(b0 + off, 16, 1024), kIdescQK, kk > 0 ? 1u : 0u);
+          mma_f16_ss(tS, make_sdesc_sw128(qa + off, 16, 1024), make_sdesc_sw128(kb + off, 16, 1024),
+                     kIdescQK, kk > 0 ? 1u : 0u);
         }
       };
-      // O_j (+)= P_j V: A = P_j from TMEM (bf16 pairs, 8 columns per 16 keys), B = V tile
-      // (MN-major: 16 keys = two 8-row groups 1024 B apart; one 64-column panel per N=64 MMA).
-      auto issue_pv = [&](int j, int vslot, bool accumulate) {
-        const uint32_t b0 = sKV + vslot * C::kStageBytes;
+      // O (+)= P V: 8 MMAs (M=128, N=DV, K=16).  A = P from TMEM (bf16 pairs: 8 columns per
+      // 16 keys).  B = V tile, MN-major: groups of 8 keys 1024 B apart (stride byte offset),
+      // 64-column panels kPanelBytes apart (leading byte offset).
+      auto issue_pv = [&](uint32_t tO, uint32_t tS, uint32_t vb, uint32_t acc_first) {
 #pragma unroll
         for (int kk = 0; kk < kBN / 16; ++kk)
-#pragma unroll
-          for (int h = 0; h < DV / 64; ++h)
-            mma_f16_ts(tO[j] + h * 64, tS[j] + kk * 8,
-                       make_sdesc_sw128(b0 + h * C::kPanelBytes + kk * 2048, 1024, 1024),
-                       kIdescPV, (accumulate || kk > 0) ? 1u : 0u);
+          mma_f16_ts(tO, tS + kk * 8, make_sdesc_sw128(vb + kk * 2048, C::kPanelBytes, 1024),
+                     kIdescPV, kk > 0 ? 1u : acc_first);
       };
-      bool ok = wait_bounded(q_full, 0, wc);
-      if (ok) ok = wait_bounded(full_bar(slot), phase, wc);
+      bool ok = wait_bounded(q_full, 0, wc) && wait_bounded(full_bar(slot), phase, wc);
       if (ok) {
         tc_fence_after_sync();
+        const uint32_t kb = sKV + slot * C::kStageBytes;
         const int ks = slot;
         next();
-        for (int j = 0; j < kQTiles; ++j) {
-          issue_qk(j, ks);
-          mma_commit(s_full(j));
-        }
+        issue_qk(tS0, sQ0, kb);
+        mma_commit(s_full(0));
+        issue_qk(tS1, sQ1, kb);
+        mma_commit(s_full(1));
         mma_commit(empty_bar(ks));
       }
       for (int n = 1; ok && n < n_kt; ++n) {
@@ -332,31 +374,42 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         ok = wait_bounded(full_bar(slot), phase, wc);
         next();
         const int ks = slot;
-        if (ok) ok = wait_bounded(full_bar(slot), phase, wc);
+        ok = ok && wait_bounded(full_bar(slot), phase, wc);
         next();
-        for (int j = 0; ok && j < kQTiles; ++j) {
-          ok = wait_bounded(p_ready(j), uint32_t(n - 1) & 1u, wc);
-          if (!ok) break;
-          tc_fence_after_sync();
-          issue_pv(j, vs, n - 1 > 0);
-          issue_qk(j, ks);
-          mma_commit(s_full(j));
-        }
-        if (ok) {
-          mma_commit(empty_bar(vs));
-          mma_commit(empty_bar(ks));
-        }
+        const uint32_t vb = sKV + vs * C::kStageBytes, kb = sKV + ks * C::kStageBytes;
+        const uint32_t par = uint32_t(n - 1) & 1u;
+        const uint32_t acc = n > 1 ? 1u : 0u;
+        ok = ok && wait_bounded(p_ready(0), par, wc);
+        if (!ok) break;
+        tc_fence_after_sync();
+        issue_pv(tO0, tS0, vb, acc);  // reads P0(n-1) before S0(n) overwrites those columns
+        issue_qk(tS0, sQ0, kb);
+        mma_commit(s_full(0));
+        ok = wait_bounded(p_ready(1), par, wc);
+        if (!ok) break;
+        tc_fence_after_sync();
+        issue_pv(tO1, tS1, vb, acc);
+        mma_commit(empty_bar(vs));
+        issue_qk(tS1, sQ1, kb);
+        mma_commit(s_full(1));
+        mma_commit(empty_bar(ks));
       }
       if (ok) {
         const int vs = slot;
-        ok = wait_bounded(full_bar(slot), phase, wc);
-        for (int j = 0; ok && j < kQTiles; ++j) {
-          ok = wait_bounded(p_ready(j), uint32_t(n_kt - 1) & 1u, wc);
-          if (!ok) break;
+        const uint32_t vb = sKV + vs * C::kStageBytes;
+        const uint32_t par = uint32_t(n_kt - 1) & 1u;
+        const uint32_t acc = n_kt > 1 ? 1u : 0u;
+        ok = wait_bounded(full_bar(slot), phase, wc) && wait_bounded(p_ready(0), par, wc);
+        if (ok) {
           tc_fence_after_sync();
-          issue_pv(j, vs, n_kt - 1 > 0);
+          issue_pv(tO0, tS0, vb, acc);
+          ok = wait_bounded(p_ready(1), par, wc);
         }
-        if (ok) mma_commit(empty_bar(vs));
+        if (ok) {
+          tc_fence_after_sync();
+          issue_pv(tO1, tS1, vb, acc);
+          mma_commit(empty_bar(vs));
+        }
       }
       // Always signal the epilogue barrier once everything issued has completed, so that the
       // TMEM is quiescent before it is freed even on the abort path.
@@ -383,72 +436,66 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       tmem_load_row128(tS, sr);
       float* s = reinterpret_cast<float*>(sr);
       const int valid = min(kBN, Nk - n * kBN);
-      // Step I: maximum of the scaled scores of this tile (max of s if c >= 0, else min).
-      float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
+      // Step I: maximum of the scaled scores of this tile (max of s if c >= 0, else of -s).
+      float tmax;
       if (valid == kBN) {
-        if (!neg) {
-#pragma unroll
-          for (int i = 0; i < kBN; i += 4) {
-            mx0 = fmaxf(mx0, s[i]);
-            mx1 = fmaxf(mx1, s[i + 1]);
-            mx2 = fmaxf(mx2, s[i + 2]);
-            mx3 = fmaxf(mx3, s[i + 3]);
-          }
-        } else {
-#pragma unroll
-          for (int i = 0; i < kBN; i += 4) {
-            mx0 = fmaxf(mx0, -s[i]);
-            mx1 = fmaxf(mx1, -s[i + 1]);
-            mx2 = fmaxf(mx2, -s[i + 2]);
-            mx3 = fmaxf(mx3, -s[i + 3]);
-          }
-        }
+        tmax = neg ? -row_max128<true>(s) : row_max128<false>(s);
       } else {
+        float mx = -INFINITY;
 #pragma unroll
         for (int i = 0; i < kBN; ++i)
-          if (i < valid) mx0 = fmaxf(mx0, neg ? -s[i] : s[i]);
+          if (i < valid) mx = fmaxf(mx, neg ? -s[i] : s[i]);
+        tmax = neg ? -mx : mx;
       }
-      const float tmax = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3));
-      const float m_tile = neg ? -c_log2 * tmax : c_log2 * tmax;  // max_k of c_log2 * s_k
+      const float m_tile = c_log2 * tmax;  // max over the tile's keys of c_log2 * s
+      bool rescale = false;  // warp-uniform
+      float alpha = 1.f;
       if (n == 0) {
         m = m_tile;
       } else {
         const bool need = m_tile > m + kRescaleLog2;
         if (__any_sync(0xffffffffu, need)) {
           const float m_new = fmaxf(m, m_tile);
-          const float alpha = ex2_approx(m - m_new);
+          alpha = ex2_approx(m - m_new);
           l *= alpha;
-          // O_j holds P V of tiles < n (complete: S_j(n) was committed after that product).
-          tmem_scale_row<DV>(tO, alpha);
           m = m_new;
+          rescale = true;
         }
       }
-      // Step II + III: p = exp2(c*s - m), row sum, P -> bf16 pairs into the S columns.
-      const float neg_m = -m;
-      float l0 = 0.f, l1 = 0.f;
-      uint32_t pk[64];
-      if (valid == kBN) {
+      // Step II + III: p = exp2(c*s - m), row sum, P -> bf16 pairs into the S columns (chunk c
+      // of 32 scores becomes 16 packed columns at column 16c; all of S is already in registers).
+      const uint64_t cc = pack_f32x2(c_log2, c_log2);
+      const uint64_t mm = pack_f32x2(-m, -m);
+      float l0 = 0.f, l1 = 0.f, l2 = 0.f, l3 = 0.f;
+      const bool full = valid == kBN;
 #pragma unroll
-        for (int i = 0; i < kBN; i += 2) {
-          const float p0 = ex2_approx(fmaf(s[i], c_log2, neg_m));
-          const float p1 = ex2_approx(fmaf(s[i + 1], c_log2, neg_m));
-          l0 += p0;
-          l1 += p1;
-          pk[i >> 1] = pack_bf16x2(p0, p1);
-        }
-      } else {
+      for (int c = 0; c < 4; ++c) {
+        uint32_t pk[16];
 #pragma unroll
-        for (int i = 0; i < kBN; i += 2) {
-          const float p0 = (i < valid) ? ex2_approx(fmaf(s[i], c_log2, neg_m)) : 0.f;
-          const float p1 = (i + 1 < valid) ? ex2_approx(fmaf(s[i + 1], c_log2, neg_m)) : 0.f;
-          l0 += p0;
-          l1 += p1;
+        for (int i = 0; i < 32; i += 4) {
+          const int k = 32 * c + i;
+          float x0, x1, x2, x3;
+          ffma2(x0, x1, s[k], s[k + 1], cc, mm);
+          ffma2(x2, x3, s[k + 2], s[k + 3], cc, mm);
+          if (!full) {
+            x0 = k < valid ? x0 : -INFINITY;
+            x1 = k + 1 < valid ? x1 : -INFINITY;
+            x2 = k + 2 < valid ? x2 : -INFINITY;
+            x3 = k + 3 < valid ? x3 : -INFINITY;
+          }
+          const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+          const float p2 = ex2_approx(x2), p3 = ex2_approx(x3);
+          fadd2(l0, l1, p0, p1);
+          fadd2(l2, l3, p2, p3);
           pk[i >> 1] = pack_bf16x2(p0, p1);
+          pk[(i >> 1) + 1] = pack_bf16x2(p2, p3);
         }
+        tmem_st_32x32b_x16(tS + 16 * c, pk);
       }
-      l += l0 + l1;
-      tmem_st_32x32b_x32(tS + 0, pk);
-      tmem_st_32x32b_x32(tS + 32, pk + 32);
+      l += (l0 + l1) + (l2 + l3);
+      // O_j holds P V of tiles < n, complete because S_j(n) was committed after that product;
+      // rescaled here, after the scores are dead, and before P_j(n) is released to the MMA.
+      if (rescale) tmem_scale_row<DV>(tO, alpha);
       tmem_wait_st();
       tc_fence_before_sync();
       mbar_arrive(p_ready(j));
