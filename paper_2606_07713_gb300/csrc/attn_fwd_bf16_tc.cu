@@ -19,19 +19,23 @@
 //     them directly.  V is the "MN-major" B operand, again as stored.
 //   * Step IV (division, Section 4.5) is applied once per row in the epilogue: O / l.
 //
-// CTA organisation (one CTA per SM: 512 TMEM columns, ~192 KB shared memory):
+// CTA organisation (one CTA per SM: 512 TMEM columns, up to ~192 KB shared memory):
 //   work item = (b*H + h, block of 256 query rows) = two 128-row Q tiles;
 //   warps 0-3: softmax + epilogue of Q tile 0; warps 4-7: same for Q tile 1
 //              (thread t of such a warpgroup owns query row t of its tile);
-//   warp 8:    TMEM allocation and the single thread that issues all tcgen05.mma;
-//   warp 9:    the single thread that issues all TMA loads.
-// K and V tiles of 128 keys stream through an NS-stage shared-memory ring in the order
-// K0, V0, K1, V1, ...; the MMA thread issues, per key tile n >= 1 and Q tile j,
-// O_j += P_j(n-1) V(n-1) and then S_j = Q_j K(n)^T, so the tensor core always has the other
-// Q tile's work while one softmax warpgroup runs.
-//
-// TMEM columns: S0 [0,128) S1 [128,256) O0 [256,256+DV) O1 [256+DV, 256+2DV); lane = row.
-//
+//   warp 8:    TMEM allocation; issues tcgen05.mma (both tiles, or tile 0 only, see below);
+//   warp 9:    the single thread that issues all TMA loads;
+//   warp 10:   issues tcgen05.mma for tile 1 when P has TMEM columns of its own.
+// K and V tiles of 128 keys stream through an NS-stage shared-memory ring.  Two schedules:
+//   d_v = 128 (TMEM: S0 S1 O0 O1): P_j is written over S_j's columns, so per key tile n >= 1
+//     the single issuing thread runs O_j += P_j(n-1) V(n-1) and then S_j = Q_j K(n)^T, tile 0
+//     then tile 1; ring order K0 V0 K1 V1 ...
+//   d_v = 64 (TMEM: S0 S1 P0 P1 O0 O1): P_j has columns of its own.  As soon as the softmax has
+//     read S_j(n) into registers, tile j's issuing thread computes S_j(n+1), and it runs
+//     O_j += P_j(n) V(n) once P_j(n) is written, so the softmax never waits for the product
+//     with V; ring order K0 K1 V0 K2 V1 ...
+// TMEM lane = row of the Q tile.
+
 // Every mbarrier wait is bounded (globaltimer); on expiry the kernel records
 // MOA_ERR_DEVICE_TIMEOUT in g_moa_bf16_status, makes every role leave its loop, and still
 // frees its TMEM before returning.
@@ -57,9 +61,10 @@ using namespace ptx;
 constexpr int kBM = 128;          // query rows per Q tile (= TMEM lanes)
 constexpr int kBN = 128;          // keys per K/V tile
 constexpr int kQTiles = 2;        // Q tiles per CTA
-constexpr int kThreads = 320;     // 8 softmax warps + MMA warp + TMA warp
-constexpr int kMmaWarp = 8;
+constexpr int kThreads = 352;     // 8 softmax warps, MMA warp (tile 0), TMA warp, MMA warp (tile 1)
+constexpr int kMmaWarp0 = 8;      // also allocates and frees TMEM
 constexpr int kLoadWarp = 9;
+constexpr int kMmaWarp1 = 10;
 constexpr int kTmemCols = 512;
 constexpr float kRescaleLog2 = 8.0f;  // lazy-rescale threshold: exponentials stay <= 2^8
 
@@ -77,11 +82,21 @@ struct Cfg {
   static constexpr int kOffQ = 0;
   static constexpr int kOffKV = kOffQ + kQTiles * kQTileBytes;
   static constexpr int kOffBar = kOffKV + kStages * kStageBytes;
-  // barriers: full[NS], empty[NS], q_full, s_full[2], p_ready[2], o_done
-  static constexpr int kNumBars = 2 * kStages + 6;
+  // P in TMEM columns of its own (d_v = 64: S0 S1 P0 P1 O0 O1 fill the 512 columns) lets the
+  // next block's scores be computed while the softmax still works on this block.  With
+  // d_v = 128 there is no room: P overwrites the S columns it came from.
+  static constexpr bool kSepP = (DV == 64);
+  // With separate P, each Q tile gets its own issuing thread (its chain of products never
+  // waits behind the other tile's).  With P aliasing S, one thread issues both tiles' products
+  // back to back, which lets the first tile's scores finish early.
+  static constexpr int kIssuers = kSepP ? 2 : 1;
+  // barriers: full[NS], empty[NS], q_full, s_full[2], p_ready[2], o_done[2], s_free[2], p_free[2]
+  static constexpr int kNumBars = 2 * kStages + 11;
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
   static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack for 1024-B alignment
-  static constexpr uint32_t kTmemS0 = 0, kTmemS1 = 128, kTmemO0 = 256, kTmemO1 = 256 + DV;
+  static constexpr uint32_t kTmemS0 = 0, kTmemS1 = 128;
+  static constexpr uint32_t kTmemP0 = kSepP ? 256 : kTmemS0, kTmemP1 = kSepP ? 320 : kTmemS1;
+  static constexpr uint32_t kTmemO0 = kSepP ? 384 : 256, kTmemO1 = kTmemO0 + DV;
   static_assert(kTmemO1 + DV <= kTmemCols, "TMEM budget");
   static_assert(kSmemBytes <= 232448, "shared memory budget");
 };
@@ -237,7 +252,9 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t q_full = bar0 + 8u * (2 * C::kStages);
   auto s_full = [&](int j) { return bar0 + 8u * (2 * C::kStages + 1 + j); };
   auto p_ready = [&](int j) { return bar0 + 8u * (2 * C::kStages + 3 + j); };
-  const uint32_t o_done = bar0 + 8u * (2 * C::kStages + 5);
+  auto o_done = [&](int j) { return bar0 + 8u * (2 * C::kStages + 5 + j); };
+  auto s_free = [&](int j) { return bar0 + 8u * (2 * C::kStages + 7 + j); };
+  auto p_free = [&](int j) { return bar0 + 8u * (2 * C::kStages + 9 + j); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
 
@@ -251,18 +268,20 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), 1);
+      mbar_init(empty_bar(s), C::kIssuers);  // one commit from each MMA issuer
     }
     mbar_init(q_full, 1);
     for (int j = 0; j < kQTiles; ++j) {
       mbar_init(s_full(j), 1);
       mbar_init(p_ready(j), 4 * 32);
+      mbar_init(o_done(j), 1);
+      mbar_init(s_free(j), 4 * 32);
+      mbar_init(p_free(j), 1);
     }
-    mbar_init(o_done, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
-  if (warp == kMmaWarp) {
+  if (warp == kMmaWarp0) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
     tmem_relinquish();
   }
@@ -287,9 +306,22 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       uint32_t phase = 0;
       uint32_t issued = 0, issued_phase = 0;  // per slot: a load was issued / its phase bit
       bool aborted = false;
+      // Ring order = the MMA issuers' consumption order: K0 V0 K1 V1 ... (P aliasing S), or
+      // K0 K1 V0 K2 V1 ... (separate P: block n+1's scores come before block n's P V).
       for (int t = 0; t < 2 * n_kt; ++t) {
-        const bool is_k = (t & 1) == 0;
-        const int n = t >> 1;
+        bool is_k;
+        int n;
+        if (!C::kSepP) {
+          is_k = (t & 1) == 0;
+          n = t >> 1;
+        } else if (t == 0) {
+          is_k = true;
+          n = 0;
+        } else {
+          const int u = t - 1, nn = u >> 1;
+          is_k = (u & 1) == 0 && nn + 1 < n_kt;
+          n = is_k ? nn + 1 : nn;
+        }
         if (!wait_bounded(empty_bar(slot), phase ^ 1u, wc)) {
           aborted = true;
           break;
@@ -320,16 +352,114 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           if (issued & (1u << sl)) wait_quiesce(full_bar(sl), (issued_phase >> sl) & 1u, wait_limit_ns);
       }
     }
-  } else if (warp == kMmaWarp) {
-    // ---------------------------------------------------------------- MMA issuer
+  } else if (warp == kMmaWarp0 || warp == kMmaWarp1) {
+    // ---------------------------------------------------------------- MMA issuers
+    // One issuing thread per Q tile, so that neither tile's products wait behind the other's.
     // Straight-line issue code: every operand of every tcgen05.mma is a loop invariant or an
-    // unrolled constant offset, so one thread keeps the tensor pipe fed.
-    if (lane == 0) {
+    // unrolled constant offset, so each thread issues at the tensor pipe's rate.
+    if constexpr (!C::kSepP) {
+      if (lane == 0 && warp == kMmaWarp0) {
+        constexpr uint32_t kIdescQK = make_idesc(kBM, kBN, false);
+        constexpr uint32_t kIdescPV = make_idesc(kBM, DV, true);
+        const uint32_t tS0 = tmem + C::kTmemS0, tS1 = tmem + C::kTmemS1;
+        const uint32_t tO0 = tmem + C::kTmemO0, tO1 = tmem + C::kTmemO1;
+        const uint32_t sQ0 = sQ, sQ1 = sQ + C::kQTileBytes;
+        int slot = 0;
+        uint32_t phase = 0;
+        auto next = [&]() {
+          if (++slot == C::kStages) {
+            slot = 0;
+            phase ^= 1u;
+          }
+        };
+        // S = Q K^T: DK/16 MMAs (M=128, N=128, K=16), both operands K-major; the k-th step is
+        // panel k/4 of the 128-byte-swizzled tile, 32 bytes further for each step inside it.
+        auto issue_qk = [&](uint32_t tS, uint32_t qa, uint32_t kb) {
+#pragma unroll
+          for (int kk = 0; kk < DK / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * C::kPanelBytes + (kk & 3) * 32;
+            mma_f16_ss(tS, make_sdesc_sw128(qa + off, 16, 1024), make_sdesc_sw128(kb + off, 16, 1024),
+                       kIdescQK, kk > 0 ? 1u : 0u);
+          }
+        };
+        // O (+)= P V: 8 MMAs (M=128, N=DV, K=16).  A = P from TMEM (bf16 pairs: 8 columns per
+        // 16 keys).  B = V tile, MN-major: groups of 8 keys 1024 B apart (stride byte offset),
+        // 64-column panels kPanelBytes apart (leading byte offset).
+        auto issue_pv = [&](uint32_t tO, uint32_t tS, uint32_t vb, uint32_t acc_first) {
+#pragma unroll
+          for (int kk = 0; kk < kBN / 16; ++kk)
+            mma_f16_ts(tO, tS + kk * 8, make_sdesc_sw128(vb + kk * 2048, C::kPanelBytes, 1024),
+                       kIdescPV, kk > 0 ? 1u : acc_first);
+        };
+        bool ok = wait_bounded(q_full, 0, wc) && wait_bounded(full_bar(slot), phase, wc);
+        if (ok) {
+          tc_fence_after_sync();
+          const uint32_t kb = sKV + slot * C::kStageBytes;
+          const int ks = slot;
+          next();
+          issue_qk(tS0, sQ0, kb);
+          mma_commit(s_full(0));
+          issue_qk(tS1, sQ1, kb);
+          mma_commit(s_full(1));
+          mma_commit(empty_bar(ks));
+        }
+        for (int n = 1; ok && n < n_kt; ++n) {
+          const int vs = slot;
+          ok = wait_bounded(full_bar(slot), phase, wc);
+          next();
+          const int ks = slot;
+          ok = ok && wait_bounded(full_bar(slot), phase, wc);
+          next();
+          const uint32_t vb = sKV + vs * C::kStageBytes, kb = sKV + ks * C::kStageBytes;
+          const uint32_t par = uint32_t(n - 1) & 1u;
+          const uint32_t acc = n > 1 ? 1u : 0u;
+          ok = ok && wait_bounded(p_ready(0), par, wc);
+          if (!ok) break;
+          tc_fence_after_sync();
+          issue_pv(tO0, tS0, vb, acc);  // reads P0(n-1) before S0(n) overwrites those columns
+          issue_qk(tS0, sQ0, kb);
+          mma_commit(s_full(0));
+          ok = wait_bounded(p_ready(1), par, wc);
+          if (!ok) break;
+          tc_fence_after_sync();
+          issue_pv(tO1, tS1, vb, acc);
+          mma_commit(empty_bar(vs));
+          issue_qk(tS1, sQ1, kb);
+          mma_commit(s_full(1));
+          mma_commit(empty_bar(ks));
+        }
+        if (ok) {
+          const int vs = slot;
+          const uint32_t vb = sKV + vs * C::kStageBytes;
+          const uint32_t par = uint32_t(n_kt - 1) & 1u;
+          const uint32_t acc = n_kt > 1 ? 1u : 0u;
+          ok = wait_bounded(full_bar(slot), phase, wc) && wait_bounded(p_ready(0), par, wc);
+          if (ok) {
+            tc_fence_after_sync();
+            issue_pv(tO0, tS0, vb, acc);
+            ok = wait_bounded(p_ready(1), par, wc);
+          }
+          if (ok) {
+            tc_fence_after_sync();
+            issue_pv(tO1, tS1, vb, acc);
+            mma_commit(empty_bar(vs));
+          }
+        }
+        // Always signal the epilogue barrier once everything issued has completed, so that the
+        // TMEM is quiescent before it is freed even on the abort path.
+        mma_commit(o_done(0));
+        mma_commit(o_done(1));
+      }
+    } else if (lane == 0) {
+      const int j = warp == kMmaWarp0 ? 0 : 1;
       constexpr uint32_t kIdescQK = make_idesc(kBM, kBN, false);
       constexpr uint32_t kIdescPV = make_idesc(kBM, DV, true);
-      const uint32_t tS0 = tmem + C::kTmemS0, tS1 = tmem + C::kTmemS1;
-      const uint32_t tO0 = tmem + C::kTmemO0, tO1 = tmem + C::kTmemO1;
-      const uint32_t sQ0 = sQ, sQ1 = sQ + C::kQTileBytes;
+      const uint32_t tS = tmem + (j ? C::kTmemS1 : C::kTmemS0);
+      const uint32_t tP = tmem + (j ? C::kTmemP1 : C::kTmemP0);
+      const uint32_t tO = tmem + (j ? C::kTmemO1 : C::kTmemO0);
+      const uint32_t sQj = sQ + j * C::kQTileBytes;
+      const uint32_t bar_s_full = s_full(j), bar_p_ready = p_ready(j), bar_s_free = s_free(j);
+      const uint32_t bar_p_free = p_free(j);
       int slot = 0;
       uint32_t phase = 0;
       auto next = [&]() {
@@ -340,80 +470,60 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       };
       // S = Q K^T: DK/16 MMAs (M=128, N=128, K=16), both operands K-major; the k-th step is
       // panel k/4 of the 128-byte-swizzled tile, 32 bytes further for each step inside it.
-      auto issue_qk = [&](uint32_t tS, uint32_t qa, uint32_t kb) {
+      auto issue_qk = [&](uint32_t kb) {
 #pragma unroll
         for (int kk = 0; kk < DK / 16; ++kk) {
           const uint32_t off = (kk >> 2) * C::kPanelBytes + (kk & 3) * 32;
-          mma_f16_ss(tS, make_sdesc_sw128(qa + off, 16, 1024), make_sdesc_sw128(kb + off, 16, 1024),
-                     kIdescQK, kk > 0 ? 1u : 0u);
+          mma_f16_ss(tS, make_sdesc_sw128(sQj + off, 16, 1024),
+                     make_sdesc_sw128(kb + off, 16, 1024), kIdescQK, kk > 0 ? 1u : 0u);
         }
       };
       // O (+)= P V: 8 MMAs (M=128, N=DV, K=16).  A = P from TMEM (bf16 pairs: 8 columns per
       // 16 keys).  B = V tile, MN-major: groups of 8 keys 1024 B apart (stride byte offset),
       // 64-column panels kPanelBytes apart (leading byte offset).
-      auto issue_pv = [&](uint32_t tO, uint32_t tS, uint32_t vb, uint32_t acc_first) {
+      auto issue_pv = [&](uint32_t vb, uint32_t acc_first) {
 #pragma unroll
         for (int kk = 0; kk < kBN / 16; ++kk)
-          mma_f16_ts(tO, tS + kk * 8, make_sdesc_sw128(vb + kk * 2048, C::kPanelBytes, 1024),
+          mma_f16_ts(tO, tP + kk * 8, make_sdesc_sw128(vb + kk * 2048, C::kPanelBytes, 1024),
                      kIdescPV, kk > 0 ? 1u : acc_first);
       };
       bool ok = wait_bounded(q_full, 0, wc) && wait_bounded(full_bar(slot), phase, wc);
       if (ok) {
         tc_fence_after_sync();
-        const uint32_t kb = sKV + slot * C::kStageBytes;
         const int ks = slot;
         next();
-        issue_qk(tS0, sQ0, kb);
-        mma_commit(s_full(0));
-        issue_qk(tS1, sQ1, kb);
-        mma_commit(s_full(1));
+        issue_qk(sKV + ks * C::kStageBytes);
+        mma_commit(bar_s_full);
         mma_commit(empty_bar(ks));
       }
-      for (int n = 1; ok && n < n_kt; ++n) {
-        const int vs = slot;
-        ok = wait_bounded(full_bar(slot), phase, wc);
-        next();
-        const int ks = slot;
-        ok = ok && wait_bounded(full_bar(slot), phase, wc);
-        next();
-        const uint32_t vb = sKV + vs * C::kStageBytes, kb = sKV + ks * C::kStageBytes;
-        const uint32_t par = uint32_t(n - 1) & 1u;
-        const uint32_t acc = n > 1 ? 1u : 0u;
-        ok = ok && wait_bounded(p_ready(0), par, wc);
-        if (!ok) break;
-        tc_fence_after_sync();
-        issue_pv(tO0, tS0, vb, acc);  // reads P0(n-1) before S0(n) overwrites those columns
-        issue_qk(tS0, sQ0, kb);
-        mma_commit(s_full(0));
-        ok = wait_bounded(p_ready(1), par, wc);
-        if (!ok) break;
-        tc_fence_after_sync();
-        issue_pv(tO1, tS1, vb, acc);
-        mma_commit(empty_bar(vs));
-        issue_qk(tS1, sQ1, kb);
-        mma_commit(s_full(1));
-        mma_commit(empty_bar(ks));
-      }
-      if (ok) {
-        const int vs = slot;
-        const uint32_t vb = sKV + vs * C::kStageBytes;
-        const uint32_t par = uint32_t(n_kt - 1) & 1u;
-        const uint32_t acc = n_kt > 1 ? 1u : 0u;
-        ok = wait_bounded(full_bar(slot), phase, wc) && wait_bounded(p_ready(0), par, wc);
-        if (ok) {
+      {
+        // P_j has columns of its own: S_j(n+1) is issued as soon as the softmax has read S_j(n),
+        // and O_j += P_j(n) V(n) once P_j(n) is written.
+        for (int n = 0; ok && n < n_kt; ++n) {
+          const uint32_t par = uint32_t(n) & 1u;
+          if (n + 1 < n_kt) {
+            const int ks = slot;
+            ok = wait_bounded(full_bar(slot), phase, wc) && wait_bounded(bar_s_free, par, wc);
+            next();
+            if (!ok) break;
+            tc_fence_after_sync();
+            issue_qk(sKV + ks * C::kStageBytes);
+            mma_commit(bar_s_full);
+            mma_commit(empty_bar(ks));
+          }
+          const int vs = slot;
+          ok = wait_bounded(full_bar(slot), phase, wc) && wait_bounded(bar_p_ready, par, wc);
+          next();
+          if (!ok) break;
           tc_fence_after_sync();
-          issue_pv(tO0, tS0, vb, acc);
-          ok = wait_bounded(p_ready(1), par, wc);
-        }
-        if (ok) {
-          tc_fence_after_sync();
-          issue_pv(tO1, tS1, vb, acc);
+          issue_pv(sKV + vs * C::kStageBytes, n > 0 ? 1u : 0u);
+          mma_commit(bar_p_free);
           mma_commit(empty_bar(vs));
         }
       }
       // Always signal the epilogue barrier once everything issued has completed, so that the
       // TMEM is quiescent before it is freed even on the abort path.
-      mma_commit(o_done);
+      mma_commit(o_done(j));
     }
   } else {
     // ---------------------------------------------------------------- softmax warpgroups
@@ -422,6 +532,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     const int row = lane_base + lane;       // query row inside the tile
     const uint32_t tS = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemS1 : C::kTmemS0);
     const uint32_t tO = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemO1 : C::kTmemO0);
+    const uint32_t tP = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemP1 : C::kTmemP0);
     const bool neg = c_log2 < 0.f;
     float m = -INFINITY;  // running maximum of c_log2 * s (log2 units)
     float l = 0.f;        // running sum of exp2(c_log2 * s - m)
@@ -434,6 +545,11 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       tc_fence_after_sync();
       uint32_t sr[128];
       tmem_load_row128(tS, sr);
+      if constexpr (C::kSepP) {
+        // S_j(n) is in registers: the MMA issuer may overwrite it with S_j(n+1).
+        tc_fence_before_sync();
+        mbar_arrive(s_free(j));
+      }
       float* s = reinterpret_cast<float*>(sr);
       const int valid = min(kBN, Nk - n * kBN);
       // Step I: maximum of the scaled scores of this tile (max of s if c >= 0, else of -s).
@@ -468,6 +584,14 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       const uint64_t mm = pack_f32x2(-m, -m);
       float l0 = 0.f, l1 = 0.f, l2 = 0.f, l3 = 0.f;
       const bool full = valid == kBN;
+      if constexpr (C::kSepP) {
+        // P_j's columns are free, and O_j may be rescaled, once O_j += P_j(n-1) V(n-1) is done.
+        if (n > 0 && !wait_bounded(p_free(j), uint32_t(n - 1) & 1u, wc)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after_sync();
+      }
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         uint32_t pk[16];
@@ -490,7 +614,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           pk[i >> 1] = pack_bf16x2(p0, p1);
           pk[(i >> 1) + 1] = pack_bf16x2(p2, p3);
         }
-        tmem_st_32x32b_x16(tS + 16 * c, pk);
+        tmem_st_32x32b_x16((C::kSepP ? tP : tS) + 16 * c, pk);
       }
       l += (l0 + l1) + (l2 + l3);
       // O_j holds P V of tiles < n, complete because S_j(n) was committed after that product;
@@ -501,7 +625,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_arrive(p_ready(j));
     }
     // Epilogue, Step IV: O / l -> bf16 -> global.
-    if (ok && wait_bounded(o_done, 0, wc)) {
+    if (ok && wait_bounded(o_done(j), 0, wc)) {
       tc_fence_after_sync();
       const float inv_l = 1.0f / l;
       const int grow = q0 + j * kBM + row;
@@ -528,10 +652,13 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   }
 
   // Teardown: wait for the tensor core to go quiet before freeing TMEM.
-  if (warp == kMmaWarp) wait_quiesce(o_done, 0, wait_limit_ns);
+  if (warp == kMmaWarp0) {
+    wait_quiesce(o_done(0), 0, wait_limit_ns);
+    wait_quiesce(o_done(1), 0, wait_limit_ns);
+  }
   tc_fence_before_sync();
   __syncthreads();
-  if (warp == kMmaWarp) {
+  if (warp == kMmaWarp0) {
     tc_fence_after_sync();
     tmem_dealloc(tmem, kTmemCols);
   }
