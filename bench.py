@@ -36,7 +36,8 @@ from paper_2606_07713_gb300 import inputs as I  # noqa: E402
 
 METRIC = "attention fwd TFLOP/s and % of GB300 bf16 peak; DRAM bytes vs DNF minimum"
 DEFAULT_WORKLOAD = 2
-PROFILE = os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b4h16n2048d64.txt")
+PROFILES = {2: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b4h16n2048d64.txt"),
+            3: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b2h32n8192d128.txt")}
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2606_07713_gb300", "csrc", f)
                   for f in ("attn_fwd_bf16_tc.cu", "ptx.cuh")]
 FLUSH_BYTES = 256 << 20
@@ -70,12 +71,12 @@ def kernel_source_hash() -> str:
     return h.hexdigest()
 
 
-def profiled_traffic() -> tuple[float | None, float | None]:
-    """(DRAM bytes per launch, ncu duration) from the committed ncu summary, if it was captured
-    from the current kernel source; (None, None) otherwise."""
+def profiled_traffic(workload: int) -> tuple[float | None, float | None]:
+    """(DRAM bytes per launch, ncu duration) from the committed ncu summary of this workload,
+    if it was captured from the current kernel source; (None, None) otherwise."""
     try:
-        text = open(PROFILE).read()
-    except OSError:
+        text = open(PROFILES[workload]).read()
+    except (KeyError, OSError):
         return None, None
     m = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", text)
     b = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
@@ -236,7 +237,7 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
         per_launch_ms = float(np.mean(kern_ms))
         achieved = flops / (per_launch_ms * 1e-3) / 1e12
         peak = float(peaks["bf16_tflops"]) if cfg.dtype == "bf16" else None
-        traffic, _ = profiled_traffic()
+        traffic, _ = profiled_traffic(cfg.cfg_id)
         line = {
             "metric": METRIC,
             "value": round(value, 2),
