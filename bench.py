@@ -145,6 +145,23 @@ class ClockSampler:
                 "power_w_max": max(power) if power else None, "reasons": sorted(reasons)}
 
 
+def reduce_max_over_ranks(values, device=None):
+    """Element-wise maximum of `values` over all ranks of the default process group (identity
+    when there is none): the slowest rank defines the whole job's time."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(list(values), dtype=torch.float64, device=device)
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
+def whole_job_tflops(flops_per_step: float, steps: int, world: int, max_ms: float) -> float:
+    """Weak scaling: every rank runs the full workload, so the job processed world * steps steps
+    in the slowest rank's time."""
+    return flops_per_step * steps * world / (max_ms * 1e-3) / 1e12
+
+
 def to_device_bf16(bits, dev):
     import torch
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
@@ -226,14 +243,11 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
     e2e_ms = float(np.sum([a.elapsed_time(b) for a, b in ev2]))
     pkg.check(pkg.get_device_status())
 
-    if world > 1:
-        t = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms, e2e_ms = float(t[0]), float(t[1])
+    total_ms, e2e_ms = reduce_max_over_ranks([total_ms, e2e_ms], device=dev)
 
     if rank == 0:
         peaks, peak_src = measured_peaks()
-        value = flops * args.steps * world / (total_ms * 1e-3) / 1e12
+        value = whole_job_tflops(flops, args.steps, world, total_ms)
         per_launch_ms = float(np.mean(kern_ms))
         achieved = flops / (per_launch_ms * 1e-3) / 1e12
         peak = float(peaks["bf16_tflops"]) if cfg.dtype == "bf16" else None
@@ -266,7 +280,7 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
                 "kernel": "attn_fwd_bf16_tc_kernel" if cfg.dtype == "bf16" else "attn_fwd_f32_cc_kernel",
             },
             "e2e": {
-                "value": round(flops * args.steps * world / (e2e_ms * 1e-3) / 1e12, 2),
+                "value": round(whole_job_tflops(flops, args.steps, world, e2e_ms), 2),
                 "unit": "TFLOP/s",
                 "h2d_bytes_per_step": int(hq.numel() * hq.element_size() + hk.numel() * hk.element_size()
                                           + hv.numel() * hv.element_size()),

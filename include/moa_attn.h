@@ -110,6 +110,19 @@ const char* moa_last_error(void);
 int moa_get_device_status(void* stream);
 
 /*
+ * moa_selftest_wait_timeout -- diagnostic for the failure path of the kernels' bounded waits
+ * (no counterpart in the paper; it exists so that timeout handling can be tested without
+ * hanging or faulting a GPU).  Launches one warp on `stream` whose thread waits, with the same
+ * bounded wait the attention kernel uses, on an mbarrier phase that nothing completes.  After
+ * limit_ns nanoseconds (0 < limit_ns <= 1e10) the wait gives up and records
+ * MOA_ERR_DEVICE_TIMEOUT in the device status word; the kernel then returns normally and the
+ * context stays usable.  Read the result with moa_get_device_status.  Asynchronous; allocates
+ * nothing.  Returns MOA_ERR_INVALID_ARG for a limit out of range, MOA_ERR_CUDA if the launch
+ * failed.
+ */
+int moa_selftest_wait_timeout(uint64_t limit_ns, void* stream);
+
+/*
  * moa_attn_flops -- floating-point operations of the two contractions,
  * 2*B*H*N_q*N_k*(d_k + d_v): the two matrix products of Eq. (attention),
  * Q K^T and the product of the weights with V (exponentials, maxima and the

@@ -15,12 +15,12 @@ import math
 
 from ._lib import (MOA_BF16, MOA_FP32, MoaError, check, lib, moa_attn_dnf_bytes,  # noqa: F401
                    moa_attn_flops, moa_attn_fwd, moa_attn_fwd_staged, moa_attn_version,
-                   moa_get_device_status, moa_last_error)
+                   moa_get_device_status, moa_last_error, moa_selftest_wait_timeout)
 
 __all__ = ["attn_fwd", "attn_fwd_staged", "get_device_status", "attn_flops", "dnf_bytes",
            "MOA_FP32", "MOA_BF16", "MoaError", "moa_attn_fwd", "moa_attn_fwd_staged",
            "moa_last_error", "moa_get_device_status", "moa_attn_flops", "moa_attn_dnf_bytes",
-           "moa_attn_version"]
+           "moa_attn_version", "moa_selftest_wait_timeout"]
 
 
 def _dtype_code(t) -> int:

@@ -42,6 +42,7 @@ SIGNATURES = {
                                            _VP]),
     "moa_last_error": (ctypes.c_char_p, []),
     "moa_get_device_status": (ctypes.c_int, [_VP]),
+    "moa_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_uint64, _VP]),
     "moa_attn_flops": (ctypes.c_double, [_I64, _I64, _I64, _I64, _I64, _I64]),
     "moa_attn_dnf_bytes": (ctypes.c_double, [_I64, _I64, _I64, _I64, _I64, _I64, ctypes.c_int]),
     "moa_attn_version": (ctypes.c_int, []),
@@ -102,6 +103,10 @@ def moa_last_error() -> str:
 
 def moa_get_device_status(stream) -> int:
     return lib().moa_get_device_status(stream)
+
+
+def moa_selftest_wait_timeout(limit_ns, stream) -> int:
+    return lib().moa_selftest_wait_timeout(limit_ns, stream)
 
 
 def moa_attn_flops(B, H, N_q, N_k, d_k, d_v) -> float:

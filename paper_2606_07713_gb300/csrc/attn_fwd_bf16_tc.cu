@@ -664,6 +664,24 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   }
 }
 
+// Failure-path self test: one thread waits, with the kernel's bounded wait, on an mbarrier
+// phase that nothing completes.  The wait must give up after limit_ns, record
+// MOA_ERR_DEVICE_TIMEOUT in the status word and return, leaving the context usable.
+__global__ void __launch_bounds__(32, 1) wait_timeout_selftest_kernel(uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_u32(&bar), 1);
+    abort_flag = 0;
+    fence_barrier_init();
+  }
+  __syncwarp();
+  if (threadIdx.x == 0) {
+    const WaitCtl wc{&abort_flag, limit_ns};
+    if (wait_bounded(smem_u32(&bar), 0, wc)) atomicExch(&g_moa_bf16_status, 0xBADu);
+  }
+}
+
 // ------------------------------------------------------------------------------------------
 // Host side
 // ------------------------------------------------------------------------------------------
@@ -761,6 +779,11 @@ int launch_attn_fwd_bf16(const AttnArgs& a, char* msg, size_t msglen) {
   snprintf(msg, msglen, "bf16 path supports d_k, d_v in {64, 128}; got d_k=%lld d_v=%lld",
            (long long)a.dk, (long long)a.dv);
   return 3;
+}
+
+cudaError_t launch_wait_timeout_selftest(uint64_t limit_ns, cudaStream_t stream) {
+  wait_timeout_selftest_kernel<<<1, 32, 0, stream>>>(limit_ns);
+  return cudaGetLastError();
 }
 
 cudaError_t bf16_read_and_clear_status(unsigned* value) {

@@ -21,6 +21,9 @@ struct AttnArgs {
 int launch_attn_fwd_f32(const AttnArgs& a, char* msg, size_t msglen);
 int launch_attn_fwd_bf16(const AttnArgs& a, char* msg, size_t msglen);
 
+// Launches the bounded-wait self test (a wait that nothing completes) on `stream`.
+cudaError_t launch_wait_timeout_selftest(uint64_t limit_ns, cudaStream_t stream);
+
 // Reads and clears the status word of the bf16 kernel's bounded waits (after a sync).
 cudaError_t bf16_read_and_clear_status(unsigned* value);
 

@@ -168,6 +168,15 @@ int moa_get_device_status(void* stream) {
   return MOA_OK;
 }
 
+int moa_selftest_wait_timeout(uint64_t limit_ns, void* stream) {
+  if (limit_ns == 0 || limit_ns > 10000000000ull)
+    return moa::fail(MOA_ERR_INVALID_ARG, "limit_ns must be in (0, 1e10]");
+  cudaError_t e = moa::launch_wait_timeout_selftest(limit_ns, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess)
+    return moa::fail(MOA_ERR_CUDA, "self-test launch: %s", cudaGetErrorString(e));
+  return MOA_OK;
+}
+
 double moa_attn_flops(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v) {
   return 2.0 * double(B) * double(H) * double(N_q) * double(N_k) * double(d_k + d_v);
 }
