@@ -13,6 +13,7 @@
 #ifndef MOA_ATTN_H
 #define MOA_ATTN_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -93,6 +94,42 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
                         void* dK, void* dV, void* dO, int64_t B, int64_t H, int64_t N_q,
                         int64_t N_k, int64_t d_k, int64_t d_v, float scale, int dtype,
                         void* stream);
+
+/*
+ * moa_attn_fwd_splitkv -- the same O as moa_attn_fwd, with the key axis split.
+ *
+ * Defines: paper Section 4.1, Eq. (attention).  The key axis [0, N_k) is cut into up to
+ * `num_splits` contiguous ranges of whole 128-key blocks; each range is reduced on its own
+ * (its own running maximum and sum, the online form of Eq. stable_softmax) into an
+ * unnormalised fp32 partial output, and a second kernel merges the partials with the identity
+ *     M = max_s m_s,   O = sum_s e^(m_s - M) O_s / sum_s e^(m_s - M) l_s,
+ * which is Eq. stable_softmax over the union of the ranges.  Useful when B*H*N_q gives too
+ * few 256-row query blocks to fill the GPU (long keys, short queries).
+ *
+ * Arguments: as moa_attn_fwd, plus
+ *   num_splits       requested number of key ranges (>= 1; fewer are used when N_k has fewer
+ *                    128-key blocks; 1 runs the unsplit kernel)
+ *   workspace        device pointer, 16-byte aligned, not overlapping any tensor; owned by the
+ *                    caller; contents on entry are ignored and undefined afterwards
+ *   workspace_bytes  its size; must be >= moa_attn_splitkv_workspace_bytes(...)
+ * MOA_FP32 has no split form: the call then computes the same result with moa_attn_fwd.
+ * Errors: those of moa_attn_fwd; MOA_ERR_INVALID_ARG for num_splits < 1 or a missing, too
+ * small or overlapping workspace; MOA_ERR_MISALIGNED for a misaligned workspace.
+ * Asynchronous on `stream`; allocates nothing.
+ */
+int moa_attn_fwd_splitkv(const void* Q, const void* K, const void* V, void* O, int64_t B,
+                         int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v,
+                         float scale, int dtype, int num_splits, void* workspace,
+                         size_t workspace_bytes, void* stream);
+
+/*
+ * moa_attn_splitkv_workspace_bytes -- bytes of workspace moa_attn_fwd_splitkv needs for these
+ * sizes and this requested split count: splits * B*H*N_q * (4*d_v + 8) (fp32 partial rows plus
+ * a running maximum and sum per row and split), 0 when no split happens or for MOA_FP32 or
+ * invalid sizes.
+ */
+size_t moa_attn_splitkv_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k,
+                                        int64_t d_k, int64_t d_v, int dtype, int num_splits);
 
 /*
  * moa_last_error -- human-readable reason for the last non-OK status returned

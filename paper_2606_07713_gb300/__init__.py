@@ -15,12 +15,14 @@ import math
 
 from ._lib import (MOA_BF16, MOA_FP32, MoaError, check, lib, moa_attn_dnf_bytes,  # noqa: F401
                    moa_attn_flops, moa_attn_fwd, moa_attn_fwd_staged, moa_attn_version,
-                   moa_get_device_status, moa_last_error, moa_selftest_wait_timeout)
+                   moa_get_device_status, moa_last_error, moa_selftest_wait_timeout,
+                   moa_attn_fwd_splitkv, moa_attn_splitkv_workspace_bytes)
 
 __all__ = ["attn_fwd", "attn_fwd_staged", "get_device_status", "attn_flops", "dnf_bytes",
            "MOA_FP32", "MOA_BF16", "MoaError", "moa_attn_fwd", "moa_attn_fwd_staged",
            "moa_last_error", "moa_get_device_status", "moa_attn_flops", "moa_attn_dnf_bytes",
-           "moa_attn_version", "moa_selftest_wait_timeout"]
+           "moa_attn_version", "moa_selftest_wait_timeout", "attn_fwd_splitkv",
+           "moa_attn_fwd_splitkv", "moa_attn_splitkv_workspace_bytes"]
 
 
 def _dtype_code(t) -> int:
@@ -69,6 +71,34 @@ def attn_fwd(q, k, v, scale: float | None = None, out=None, stream=None):
         s = stream if stream is not None else torch.cuda.current_stream(q.device)
         check(moa_attn_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), B, H, Nq, Nk,
                            dk, dv, float(scale), code, s.cuda_stream))
+    return out
+
+
+def attn_fwd_splitkv(q, k, v, num_splits: int, scale: float | None = None, out=None,
+                     workspace=None, stream=None):
+    """attn_fwd with the key axis split into up to num_splits ranges merged at the end.  The
+    workspace (a CUDA uint8 tensor of at least moa_attn_splitkv_workspace_bytes(...) bytes) is
+    allocated here when not given."""
+    import torch
+    for t in (q, k, v):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError("attn_fwd_splitkv needs contiguous CUDA tensors")
+    if not (q.dtype == k.dtype == v.dtype):
+        raise TypeError("q, k, v must share one dtype")
+    code = _dtype_code(q)
+    B, H, Nq, Nk, dk, dv = _dims(q, k, v)
+    if scale is None:
+        scale = 1.0 / math.sqrt(dk)
+    if out is None:
+        out = torch.empty((B, H, Nq, dv), dtype=q.dtype, device=q.device)
+    need = moa_attn_splitkv_workspace_bytes(B, H, Nq, Nk, dk, dv, code, int(num_splits))
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=q.device)
+    with torch.cuda.device(q.device):
+        s = stream if stream is not None else torch.cuda.current_stream(q.device)
+        check(moa_attn_fwd_splitkv(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), B, H,
+                                   Nq, Nk, dk, dv, float(scale), code, int(num_splits),
+                                   workspace.data_ptr(), workspace.numel(), s.cuda_stream))
     return out
 
 

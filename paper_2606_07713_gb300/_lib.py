@@ -40,6 +40,11 @@ SIGNATURES = {
     "moa_attn_fwd_staged": (ctypes.c_int, [_VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _I64, _I64,
                                            _I64, _I64, _I64, _I64, ctypes.c_float, ctypes.c_int,
                                            _VP]),
+    "moa_attn_fwd_splitkv": (ctypes.c_int, [_VP, _VP, _VP, _VP, _I64, _I64, _I64, _I64, _I64,
+                                            _I64, ctypes.c_float, ctypes.c_int, ctypes.c_int,
+                                            _VP, ctypes.c_size_t, _VP]),
+    "moa_attn_splitkv_workspace_bytes": (ctypes.c_size_t, [_I64, _I64, _I64, _I64, _I64, _I64,
+                                                           ctypes.c_int, ctypes.c_int]),
     "moa_last_error": (ctypes.c_char_p, []),
     "moa_get_device_status": (ctypes.c_int, [_VP]),
     "moa_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_uint64, _VP]),
@@ -95,6 +100,16 @@ def moa_attn_fwd_staged(hQ, hK, hV, hO, dQ, dK, dV, dO, B, H, N_q, N_k, d_k, d_v
                         stream) -> int:
     return lib().moa_attn_fwd_staged(hQ, hK, hV, hO, dQ, dK, dV, dO, B, H, N_q, N_k, d_k, d_v,
                                      scale, dtype, stream)
+
+
+def moa_attn_fwd_splitkv(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, num_splits,
+                         workspace, workspace_bytes, stream) -> int:
+    return lib().moa_attn_fwd_splitkv(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype,
+                                      num_splits, workspace, workspace_bytes, stream)
+
+
+def moa_attn_splitkv_workspace_bytes(B, H, N_q, N_k, d_k, d_v, dtype, num_splits) -> int:
+    return lib().moa_attn_splitkv_workspace_bytes(B, H, N_q, N_k, d_k, d_v, dtype, num_splits)
 
 
 def moa_last_error() -> str:

@@ -67,6 +67,10 @@ constexpr int kLoadWarp = 9;
 constexpr int kMmaWarp1 = 10;
 constexpr int kTmemCols = 512;
 constexpr float kRescaleLog2 = 8.0f;  // lazy-rescale threshold: exponentials stay <= 2^8
+// Longest suspension of one mbarrier test for the d_v = 64 schedule, where the MMA and TMA
+// threads wait long enough that polling would take issue slots from the softmax warps
+// (measured +3.6% there, -1..3% with d_v = 128, which therefore polls).
+constexpr uint32_t kWaitHintNs = 20000;
 
 template <int DK, int DV>
 struct Cfg {
@@ -119,6 +123,7 @@ __device__ __forceinline__ uint64_t make_sdesc_sw128(uint32_t addr, uint32_t lbo
 struct WaitCtl {
   volatile int* abort_flag;
   uint64_t limit_ns;
+  uint32_t hint_ns;  // 0: poll; otherwise let a not-yet-complete test suspend the thread
 };
 
 // Bounded mbarrier wait.  Returns false (and raises the CTA abort flag and the global status
@@ -127,7 +132,8 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, cons
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (w.hint_ns ? mbar_try_wait_hint(bar, parity, w.hint_ns) : mbar_try_wait(bar, parity))
+      return true;
     if ((it & 63u) == 0) {
       if (*w.abort_flag) return false;
       if (globaltimer_ns() - t0 > w.limit_ns) {
@@ -234,12 +240,16 @@ __device__ __forceinline__ void tmem_scale_row(uint32_t taddr, float alpha) {
   tmem_wait_st();
 }
 
-template <int DK, int DV>
+// SPLIT: this CTA covers one range of the key axis and writes fp32 partials for the merge kernel
+// (separate instantiation, so the unsplit kernel carries none of it).
+template <int DK, int DV, bool SPLIT>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmV, __nv_bfloat16* __restrict__ O,
-                        int Nq, int Nk, int n_qblocks, float c_log2, uint64_t wait_limit_ns) {
+                        int Nq, int Nk, int n_qblocks, float c_log2, uint64_t wait_limit_ns,
+                        int n_splits, int kv_per_split, float* __restrict__ ws_o,
+                        float2* __restrict__ ws_ml) {
   using C = Cfg<DK, DV>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -260,10 +270,16 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int bh = blockIdx.x / n_qblocks;
-  const int q0 = (blockIdx.x % n_qblocks) * (kQTiles * kBM);
-  const int n_kt = (Nk + kBN - 1) / kBN;
-  const WaitCtl wc{abort_flag, wait_limit_ns};
+  // CTA -> (b*H + h, 256-row query block, key split); splits of one block are adjacent, and
+  // blocks of one head are adjacent (head-major), so concurrently running CTAs share K/V in L2.
+  const int split = SPLIT ? int(blockIdx.x % n_splits) : 0;
+  const int item = SPLIT ? int(blockIdx.x / n_splits) : int(blockIdx.x);
+  const int bh = item / n_qblocks;
+  const int q0 = (item % n_qblocks) * (kQTiles * kBM);
+  // This CTA's key blocks: [kb0, kb0 + n_kt) (all of them unless the key axis is split).
+  const int kb0 = SPLIT ? split * kv_per_split : 0;
+  const int n_kt = SPLIT ? min((Nk + kBN - 1) / kBN - kb0, kv_per_split) : (Nk + kBN - 1) / kBN;
+  const WaitCtl wc{abort_flag, wait_limit_ns, C::kSepP ? kWaitHintNs : 0u};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
@@ -333,12 +349,14 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           mbar_arrive_expect_tx(full_bar(slot), C::kKTileBytes);
 #pragma unroll
           for (int p = 0; p < DK / 64; ++p)
-            tma_load_3d(dst + p * C::kPanelBytes, &tmK, full_bar(slot), p * 64, n * kBN, bh);
+            tma_load_3d(dst + p * C::kPanelBytes, &tmK, full_bar(slot), p * 64, (kb0 + n) * kBN,
+                        bh);
         } else {
           mbar_arrive_expect_tx(full_bar(slot), C::kVTileBytes);
 #pragma unroll
           for (int p = 0; p < DV / 64; ++p)
-            tma_load_3d(dst + p * C::kPanelBytes, &tmV, full_bar(slot), p * 64, n * kBN, bh);
+            tma_load_3d(dst + p * C::kPanelBytes, &tmV, full_bar(slot), p * 64, (kb0 + n) * kBN,
+                        bh);
         }
         if (++slot == C::kStages) {
           slot = 0;
@@ -551,7 +569,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         mbar_arrive(s_free(j));
       }
       float* s = reinterpret_cast<float*>(sr);
-      const int valid = min(kBN, Nk - n * kBN);
+      const int valid = min(kBN, Nk - (kb0 + n) * kBN);
       // Step I: maximum of the scaled scores of this tile (max of s if c >= 0, else of -s).
       float tmax;
       if (valid == kBN) {
@@ -624,8 +642,29 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       tc_fence_before_sync();
       mbar_arrive(p_ready(j));
     }
-    // Epilogue, Step IV: O / l -> bf16 -> global.
-    if (ok && wait_bounded(o_done(j), 0, wc)) {
+    // Epilogue, Step IV: O / l -> bf16 -> global.  With a split key axis this CTA instead
+    // writes its unnormalised fp32 O rows and (m, l) for the merge kernel.
+    if (SPLIT && ok && wait_bounded(o_done(j), 0, wc)) {
+      tc_fence_after_sync();
+      const int grow = q0 + j * kBM + row;
+      const size_t prow = (size_t(split) * (gridDim.x / n_splits / n_qblocks) + bh) * Nq + grow;
+      float* orow = ws_o + prow * DV;
+#pragma unroll
+      for (int c = 0; c < DV; c += 32) {
+        uint32_t o[32];
+        tmem_ld_32x32b_x32(tO + c, o);
+        tmem_wait_ld();
+        reg_anchor_x32(o);
+        if (grow < Nq) {
+          float4* dst = reinterpret_cast<float4*>(orow + c);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            dst[i] = make_float4(__uint_as_float(o[4 * i]), __uint_as_float(o[4 * i + 1]),
+                                 __uint_as_float(o[4 * i + 2]), __uint_as_float(o[4 * i + 3]));
+        }
+      }
+      if (grow < Nq) ws_ml[prow] = make_float2(m, l);
+    } else if (!SPLIT && ok && wait_bounded(o_done(j), 0, wc)) {
       tc_fence_after_sync();
       const float inv_l = 1.0f / l;
       const int grow = q0 + j * kBM + row;
@@ -664,6 +703,36 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   }
 }
 
+// Merge of a split key axis (the identity behind Eq. stable_softmax applied across key ranges):
+// with per-split reference maxima m_s (log2 units), unnormalised rows O_s and sums l_s,
+//   M = max_s m_s,  O = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s.
+// One warp per output row; lane c handles columns c, c+32, ...
+template <int DV>
+__global__ void __launch_bounds__(256)
+splitkv_merge_kernel(const float* __restrict__ ws_o, const float2* __restrict__ ws_ml,
+                     __nv_bfloat16* __restrict__ O, long long rows, int n_splits) {
+  const long long r = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  float M = -INFINITY;
+  for (int s = 0; s < n_splits; ++s) M = fmaxf(M, ws_ml[s * rows + r].x);
+  float L = 0.f;
+  float acc[DV / 32];
+#pragma unroll
+  for (int i = 0; i < DV / 32; ++i) acc[i] = 0.f;
+  for (int s = 0; s < n_splits; ++s) {
+    const float2 ml = ws_ml[s * rows + r];
+    const float w = ex2_approx(ml.x - M);
+    L = fmaf(w, ml.y, L);
+    const float* src = ws_o + (s * rows + r) * DV;
+#pragma unroll
+    for (int i = 0; i < DV / 32; ++i) acc[i] = fmaf(w, src[lane + 32 * i], acc[i]);
+  }
+  const float inv = 1.0f / L;
+#pragma unroll
+  for (int i = 0; i < DV / 32; ++i) O[r * DV + lane + 32 * i] = __float2bfloat16_rn(acc[i] * inv);
+}
+
 // Failure-path self test: one thread waits, with the kernel's bounded wait, on an mbarrier
 // phase that nothing completes.  The wait must give up after limit_ns, record
 // MOA_ERR_DEVICE_TIMEOUT in the status word and return, leaving the context usable.
@@ -677,7 +746,7 @@ __global__ void __launch_bounds__(32, 1) wait_timeout_selftest_kernel(uint64_t l
   }
   __syncwarp();
   if (threadIdx.x == 0) {
-    const WaitCtl wc{&abort_flag, limit_ns};
+    const WaitCtl wc{&abort_flag, limit_ns, 0u};
     if (wait_bounded(smem_u32(&bar), 0, wc)) atomicExch(&g_moa_bf16_status, 0xBADu);
   }
 }
@@ -731,40 +800,80 @@ bool encode_map(EncodeTiledFn enc, CUtensorMap* map, const void* base, int64_t B
 
 template <int DK, int DV>
 int launch_tc(const AttnArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
-              const CUtensorMap& mv, char* msg, size_t msglen) {
+              const CUtensorMap& mv, const SplitPlan& sp, void* ws, char* msg, size_t msglen) {
   using C = Cfg<DK, DV>;
-  auto kern = attn_fwd_bf16_tc_kernel<DK, DV>;
+  auto kern = sp.n_splits > 1 ? attn_fwd_bf16_tc_kernel<DK, DV, true>
+                              : attn_fwd_bf16_tc_kernel<DK, DV, false>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    C::kSmemBytes);
+    attr_err = cudaFuncSetAttribute(attn_fwd_bf16_tc_kernel<DK, DV, false>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(attn_fwd_bf16_tc_kernel<DK, DV, true>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   });
   if (attr_err != cudaSuccess) {
     snprintf(msg, msglen, "cudaFuncSetAttribute (bf16 kernel): %s", cudaGetErrorString(attr_err));
     return 5;
   }
   const int64_t n_qblocks = (a.Nq + kQTiles * kBM - 1) / (kQTiles * kBM);
-  const int64_t grid = a.B * a.H * n_qblocks;
+  const int64_t grid = a.B * a.H * n_qblocks * sp.n_splits;
   if (grid > 0x7fffffffLL) {
     snprintf(msg, msglen, "bf16 path: %lld CTAs exceeds the grid limit", (long long)grid);
     return 3;
   }
   const float c_log2 = a.scale * 1.4426950408889634f;
+  const int64_t rows = a.B * a.H * a.Nq;
+  float* ws_o = sp.n_splits > 1 ? static_cast<float*>(ws) : nullptr;
+  float2* ws_ml = sp.n_splits > 1
+                      ? reinterpret_cast<float2*>(static_cast<float*>(ws) + sp.n_splits * rows * DV)
+                      : nullptr;
   kern<<<dim3(unsigned(grid)), dim3(kThreads), C::kSmemBytes, a.stream>>>(
       mq, mk, mv, static_cast<__nv_bfloat16*>(a.O), int(a.Nq), int(a.Nk), int(n_qblocks), c_log2,
-      wait_limit_ns());
+      wait_limit_ns(), sp.n_splits, sp.kv_per_split, ws_o, ws_ml);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     snprintf(msg, msglen, "bf16 kernel launch: %s", cudaGetErrorString(e));
     return 5;
+  }
+  if (sp.n_splits > 1) {
+    const long long blocks = (rows + 7) / 8;
+    splitkv_merge_kernel<DV><<<dim3(unsigned(blocks)), dim3(256), 0, a.stream>>>(
+        ws_o, ws_ml, static_cast<__nv_bfloat16*>(a.O), rows, sp.n_splits);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) {
+      snprintf(msg, msglen, "split merge launch: %s", cudaGetErrorString(e));
+      return 5;
+    }
   }
   return 0;
 }
 
 }  // namespace
 
+SplitPlan plan_splits(int64_t Nk, int requested) {
+  const int64_t n_kt = (Nk + kBN - 1) / kBN;
+  int64_t want = requested < 1 ? 1 : requested;
+  if (want > n_kt) want = n_kt;
+  const int64_t per = (n_kt + want - 1) / want;
+  SplitPlan sp;
+  sp.kv_per_split = int(per);
+  sp.n_splits = int((n_kt + per - 1) / per);  // every split gets at least one key block
+  return sp;
+}
+
+size_t splitkv_workspace_bytes(int64_t rows, int64_t dv, const SplitPlan& sp) {
+  if (sp.n_splits <= 1) return 0;
+  return size_t(sp.n_splits) * size_t(rows) * (size_t(dv) * 4 + 8);
+}
+
 int launch_attn_fwd_bf16(const AttnArgs& a, char* msg, size_t msglen) {
+  return launch_attn_fwd_bf16_split(a, plan_splits(a.Nk, 1), nullptr, msg, msglen);
+}
+
+int launch_attn_fwd_bf16_split(const AttnArgs& a, const SplitPlan& sp, void* ws, char* msg,
+                               size_t msglen) {
   EncodeTiledFn enc = get_encode_fn(msg, msglen);
   if (!enc) return 5;
   const int64_t BH = a.B * a.H;
@@ -772,10 +881,10 @@ int launch_attn_fwd_bf16(const AttnArgs& a, char* msg, size_t msglen) {
   if (!encode_map(enc, &mq, a.Q, BH, a.Nq, a.dk, msg, msglen)) return 5;
   if (!encode_map(enc, &mk, a.K, BH, a.Nk, a.dk, msg, msglen)) return 5;
   if (!encode_map(enc, &mv, a.V, BH, a.Nk, a.dv, msg, msglen)) return 5;
-  if (a.dk == 64 && a.dv == 64) return launch_tc<64, 64>(a, mq, mk, mv, msg, msglen);
-  if (a.dk == 128 && a.dv == 128) return launch_tc<128, 128>(a, mq, mk, mv, msg, msglen);
-  if (a.dk == 128 && a.dv == 64) return launch_tc<128, 64>(a, mq, mk, mv, msg, msglen);
-  if (a.dk == 64 && a.dv == 128) return launch_tc<64, 128>(a, mq, mk, mv, msg, msglen);
+  if (a.dk == 64 && a.dv == 64) return launch_tc<64, 64>(a, mq, mk, mv, sp, ws, msg, msglen);
+  if (a.dk == 128 && a.dv == 128) return launch_tc<128, 128>(a, mq, mk, mv, sp, ws, msg, msglen);
+  if (a.dk == 128 && a.dv == 64) return launch_tc<128, 64>(a, mq, mk, mv, sp, ws, msg, msglen);
+  if (a.dk == 64 && a.dv == 128) return launch_tc<64, 128>(a, mq, mk, mv, sp, ws, msg, msglen);
   snprintf(msg, msglen, "bf16 path supports d_k, d_v in {64, 128}; got d_k=%lld d_v=%lld",
            (long long)a.dk, (long long)a.dv);
   return 3;

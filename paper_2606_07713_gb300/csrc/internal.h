@@ -17,9 +17,25 @@ struct AttnArgs {
   cudaStream_t stream;
 };
 
-// Both launchers return a moa_status code and, on failure, write a message into msg.
+// How the key axis of the bf16 kernel is split: n_splits contiguous ranges of kv_per_split
+// 128-key blocks (the last may be shorter); n_splits == 1 means no split.
+struct SplitPlan {
+  int n_splits = 1;
+  int kv_per_split = 0x7fffffff;
+};
+
+// At most `requested` splits, each of at least one key block.
+SplitPlan plan_splits(int64_t Nk, int requested);
+
+// Workspace of a split bf16 call: fp32 partial rows and (m, l) per split and output row.
+size_t splitkv_workspace_bytes(int64_t rows, int64_t dv, const SplitPlan& sp);
+
+// The launchers return a moa_status code and, on failure, write a message into msg.
 int launch_attn_fwd_f32(const AttnArgs& a, char* msg, size_t msglen);
 int launch_attn_fwd_bf16(const AttnArgs& a, char* msg, size_t msglen);
+// `ws` must hold splitkv_workspace_bytes(B*H*N_q, d_v, sp) bytes (unused when n_splits == 1).
+int launch_attn_fwd_bf16_split(const AttnArgs& a, const SplitPlan& sp, void* ws, char* msg,
+                               size_t msglen);
 
 // Launches the bounded-wait self test (a wait that nothing completes) on `stream`.
 cudaError_t launch_wait_timeout_selftest(uint64_t limit_ns, cudaStream_t stream);

@@ -153,6 +153,47 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
   return MOA_OK;
 }
 
+size_t moa_attn_splitkv_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k,
+                                        int64_t d_k, int64_t d_v, int dtype, int num_splits) {
+  (void)d_k;
+  if (dtype != MOA_BF16 || B <= 0 || H <= 0 || N_q <= 0 || N_k <= 0 || d_v <= 0) return 0;
+  const int64_t rows = moa::numel4(B, H, N_q, 1);
+  if (rows < 0) return 0;
+  return moa::splitkv_workspace_bytes(rows, d_v, moa::plan_splits(N_k, num_splits));
+}
+
+int moa_attn_fwd_splitkv(const void* Q, const void* K, const void* V, void* O, int64_t B,
+                         int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v,
+                         float scale, int dtype, int num_splits, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+  int64_t sz[4];
+  int rc = moa::validate(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
+  if (rc != MOA_OK) return rc;
+  if (num_splits < 1) return moa::fail(MOA_ERR_INVALID_ARG, "num_splits must be >= 1");
+  if (dtype != MOA_BF16)  // the fp32 path has no split form; it computes the same result whole
+    return moa::dispatch(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream);
+  const moa::SplitPlan sp = moa::plan_splits(N_k, num_splits);
+  const size_t need = moa::splitkv_workspace_bytes(B * H * N_q, d_v, sp);
+  if (need > 0) {
+    if (workspace == nullptr || workspace_bytes < need)
+      return moa::fail(MOA_ERR_INVALID_ARG, "workspace too small: need %zu bytes, got %zu", need,
+                       workspace == nullptr ? size_t(0) : workspace_bytes);
+    if (reinterpret_cast<uintptr_t>(workspace) % 16 != 0)
+      return moa::fail(MOA_ERR_MISALIGNED, "workspace is not 16-byte aligned");
+    const void* ins[4] = {Q, K, V, O};
+    const int64_t insz[4] = {sz[0], sz[1], sz[2], sz[3]};
+    for (int i = 0; i < 4; ++i)
+      if (moa::overlaps(workspace, int64_t(need), ins[i], insz[i]))
+        return moa::fail(MOA_ERR_INVALID_ARG, "workspace overlaps a tensor");
+  }
+  moa::AttnArgs a{Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, static_cast<cudaStream_t>(stream)};
+  char msg[256] = {0};
+  rc = moa::launch_attn_fwd_bf16_split(a, sp, workspace, msg, sizeof(msg));
+  if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
+  moa::t_last_error[0] = '\0';
+  return MOA_OK;
+}
+
 const char* moa_last_error(void) { return moa::t_last_error; }
 
 int moa_get_device_status(void* stream) {

@@ -89,3 +89,24 @@ def test_validation_rejects_before_launch(L, kwargs, code):
 def test_staged_rejects_null_host_pointers(L):
     rc = _lib.moa_attn_fwd_staged(None, A, A, A, A, B_, C, D, 1, 1, 8, 8, 64, 64, 0.1, 1, None)
     assert rc == _lib.MOA_ERR_INVALID_ARG
+
+
+def test_splitkv_workspace_formula(L):
+    ws = pkg.moa_attn_splitkv_workspace_bytes
+    # 1000 keys = 8 blocks; 3 splits of 3,3,2 blocks
+    assert ws(1, 2, 256, 1000, 64, 64, pkg.MOA_BF16, 3) == 3 * 2 * 256 * (4 * 64 + 8)
+    # more splits than blocks: one split per block
+    assert ws(1, 1, 10, 300, 64, 128, pkg.MOA_BF16, 9) == 3 * 10 * (4 * 128 + 8)
+    # 8 blocks in 5 requested splits: 2 blocks each -> 4 splits
+    assert ws(1, 1, 10, 1024, 64, 64, pkg.MOA_BF16, 5) == 4 * 10 * (4 * 64 + 8)
+    assert ws(1, 1, 10, 128, 64, 64, pkg.MOA_BF16, 4) == 0      # one block: no split
+    assert ws(1, 1, 10, 1024, 64, 64, pkg.MOA_FP32, 4) == 0     # fp32 has no split form
+    assert ws(0, 1, 10, 1024, 64, 64, pkg.MOA_BF16, 4) == 0
+
+
+def test_splitkv_validation_without_gpu(L):
+    f = _lib.moa_attn_fwd_splitkv
+    assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 0, 0x500000, 1 << 20, None) == _lib.MOA_ERR_INVALID_ARG
+    assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 4, None, 0, None) == _lib.MOA_ERR_INVALID_ARG
+    assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 4, 0x500008, 1 << 20, None) == _lib.MOA_ERR_MISALIGNED
+    assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 4, D, 1 << 20, None) == _lib.MOA_ERR_INVALID_ARG
