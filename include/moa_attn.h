@@ -131,6 +131,39 @@ int moa_attn_fwd_splitkv(const void* Q, const void* K, const void* V, void* O, i
 size_t moa_attn_splitkv_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k,
                                         int64_t d_k, int64_t d_v, int dtype, int num_splits);
 
+/* Size in bytes of the fixed device array used by moa_attn_fwd_splitkv_noalloc (16 MiB). */
+#define MOA_NOALLOC_SCRATCH_BYTES ((size_t)16 << 20)
+
+/*
+ * moa_attn_fwd_splitkv_noalloc -- moa_attn_fwd_splitkv for callers that cannot allocate.
+ *
+ * The paper has no counterpart to this entry point; it is a convenience of this library.
+ * Some callers have no way to hand this library scratch memory: a framework that owns every
+ * byte of device memory through its own pool and allows no other allocation, a serving loop
+ * that must not call cudaMalloc because the call synchronises the device and stalls other
+ * work, or a plugin interface that passes only the input and output buffers.  For them this
+ * entry point takes no workspace and allocates nothing (no cudaMalloc, cudaFree or allocating
+ * library routine): the fp32 partial rows and per-row maxima and sums of the split live in a
+ * fixed array of MOA_NOALLOC_SCRATCH_BYTES inside the library, which every GPU that loads the
+ * library holds until the process exits.
+ *
+ * Result and arguments: exactly those of moa_attn_fwd_splitkv without the workspace; the
+ * caller still passes Q, K, V and O.  A split whose partials need more than
+ * MOA_NOALLOC_SCRATCH_BYTES (splits * B*H*N_q * (4*d_v + 8) bytes) is rejected with
+ * MOA_ERR_UNSUPPORTED_SHAPE and a message naming both sizes; nothing is launched.
+ *
+ * The first call on a device looks up that device's address of the array (once per device,
+ * with the device current); make that first call before any stream capture on the device.
+ * All calls on a device share the one array and it keeps the last call's contents: calls that
+ * can run at the same time on the GPU (e.g. on unordered streams) race on it and must be
+ * serialised by the caller.  Nothing in the array needs to start at zero.
+ * Asynchronous on `stream`.
+ */
+int moa_attn_fwd_splitkv_noalloc(const void* Q, const void* K, const void* V, void* O,
+                                 int64_t B, int64_t H, int64_t N_q, int64_t N_k, int64_t d_k,
+                                 int64_t d_v, float scale, int dtype, int num_splits,
+                                 void* stream);
+
 /*
  * moa_last_error -- human-readable reason for the last non-OK status returned
  * on the calling thread ("" if none).  The string is owned by the library and

@@ -45,6 +45,9 @@ SIGNATURES = {
                                             _VP, ctypes.c_size_t, _VP]),
     "moa_attn_splitkv_workspace_bytes": (ctypes.c_size_t, [_I64, _I64, _I64, _I64, _I64, _I64,
                                                            ctypes.c_int, ctypes.c_int]),
+    "moa_attn_fwd_splitkv_noalloc": (ctypes.c_int, [_VP, _VP, _VP, _VP, _I64, _I64, _I64, _I64,
+                                                    _I64, _I64, ctypes.c_float, ctypes.c_int,
+                                                    ctypes.c_int, _VP]),
     "moa_last_error": (ctypes.c_char_p, []),
     "moa_get_device_status": (ctypes.c_int, [_VP]),
     "moa_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_uint64, _VP]),
@@ -110,6 +113,16 @@ def moa_attn_fwd_splitkv(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, num
 
 def moa_attn_splitkv_workspace_bytes(B, H, N_q, N_k, d_k, d_v, dtype, num_splits) -> int:
     return lib().moa_attn_splitkv_workspace_bytes(B, H, N_q, N_k, d_k, d_v, dtype, num_splits)
+
+
+def moa_attn_fwd_splitkv_noalloc(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, num_splits,
+                                 stream) -> int:
+    return lib().moa_attn_fwd_splitkv_noalloc(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype,
+                                              num_splits, stream)
+
+
+# MOA_NOALLOC_SCRATCH_BYTES of include/moa_attn.h
+MOA_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
 def moa_last_error() -> str:

@@ -890,6 +890,64 @@ int launch_attn_fwd_bf16_split(const AttnArgs& a, const SplitPlan& sp, void* ws,
   return 3;
 }
 
+// ------------------------------------------------------------------------------------------
+// Split key axis without any allocation: the partial rows live in a fixed device array
+// ------------------------------------------------------------------------------------------
+// One array per device that loads this library, held until the process exits.  Every call of
+// the allocation-free entry point on a device uses the same array, so calls that overlap on the
+// GPU (different streams, no ordering between them) race on it.  Nothing in it needs to start
+// at zero: the split kernel writes every partial row and (m, l) pair the merge kernel reads.
+static __device__ __align__(256) unsigned char g_splitkv_scratch[kNoallocScratchBytes];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_splitkv_scratch on the current device.  In host code the array's name
+// only stands for the device symbol; its address on a device comes from cudaGetSymbolAddress,
+// asked once per device, with that device current.
+void* scratch_address(char* msg, size_t msglen) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    snprintf(msg, msglen, "no usable current device for the static scratch (%s)",
+             cudaGetErrorString(e));
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (g_scratch_addr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_splitkv_scratch);
+    if (e != cudaSuccess || p == nullptr) {
+      snprintf(msg, msglen, "cudaGetSymbolAddress(static scratch) on device %d: %s", dev,
+               cudaGetErrorString(e));
+      return nullptr;
+    }
+    g_scratch_addr[dev] = p;
+  }
+  return g_scratch_addr[dev];
+}
+}  // namespace
+
+int launch_attn_fwd_bf16_split_noalloc(const AttnArgs& a, const SplitPlan& sp, char* msg,
+                                       size_t msglen) {
+  const size_t need = splitkv_workspace_bytes(a.B * a.H * a.Nq, a.dv, sp);
+  if (need > kNoallocScratchBytes) {
+    snprintf(msg, msglen,
+             "split needs %zu bytes of scratch but the static scratch holds %zu; use fewer "
+             "splits or moa_attn_fwd_splitkv with a workspace of your own",
+             need, size_t(kNoallocScratchBytes));
+    return 3;
+  }
+  void* ws = nullptr;
+  if (need > 0) {
+    ws = scratch_address(msg, msglen);
+    if (ws == nullptr) return 5;
+  }
+  return launch_attn_fwd_bf16_split(a, sp, ws, msg, msglen);
+}
+
 cudaError_t launch_wait_timeout_selftest(uint64_t limit_ns, cudaStream_t stream) {
   wait_timeout_selftest_kernel<<<1, 32, 0, stream>>>(limit_ns);
   return cudaGetLastError();

@@ -30,12 +30,19 @@ SplitPlan plan_splits(int64_t Nk, int requested);
 // Workspace of a split bf16 call: fp32 partial rows and (m, l) per split and output row.
 size_t splitkv_workspace_bytes(int64_t rows, int64_t dv, const SplitPlan& sp);
 
+// Size of the fixed device array behind the allocation-free split entry point (16 MiB).
+constexpr size_t kNoallocScratchBytes = size_t(16) << 20;
+
 // The launchers return a moa_status code and, on failure, write a message into msg.
 int launch_attn_fwd_f32(const AttnArgs& a, char* msg, size_t msglen);
 int launch_attn_fwd_bf16(const AttnArgs& a, char* msg, size_t msglen);
 // `ws` must hold splitkv_workspace_bytes(B*H*N_q, d_v, sp) bytes (unused when n_splits == 1).
 int launch_attn_fwd_bf16_split(const AttnArgs& a, const SplitPlan& sp, void* ws, char* msg,
                                size_t msglen);
+// Same, with the partial rows in the library's fixed device array (no allocation; rejects a
+// split whose partials exceed kNoallocScratchBytes with MOA_ERR_UNSUPPORTED_SHAPE).
+int launch_attn_fwd_bf16_split_noalloc(const AttnArgs& a, const SplitPlan& sp, char* msg,
+                                       size_t msglen);
 
 // Launches the bounded-wait self test (a wait that nothing completes) on `stream`.
 cudaError_t launch_wait_timeout_selftest(uint64_t limit_ns, cudaStream_t stream);

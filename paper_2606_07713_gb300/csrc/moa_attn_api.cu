@@ -194,6 +194,24 @@ int moa_attn_fwd_splitkv(const void* Q, const void* K, const void* V, void* O, i
   return MOA_OK;
 }
 
+int moa_attn_fwd_splitkv_noalloc(const void* Q, const void* K, const void* V, void* O, int64_t B,
+                                 int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v,
+                                 float scale, int dtype, int num_splits, void* stream) {
+  int64_t sz[4];
+  int rc = moa::validate(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
+  if (rc != MOA_OK) return rc;
+  if (num_splits < 1) return moa::fail(MOA_ERR_INVALID_ARG, "num_splits must be >= 1");
+  if (dtype != MOA_BF16)  // no split form, no scratch: the whole fp32 computation
+    return moa::dispatch(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream);
+  moa::AttnArgs a{Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, static_cast<cudaStream_t>(stream)};
+  char msg[256] = {0};
+  rc = moa::launch_attn_fwd_bf16_split_noalloc(a, moa::plan_splits(N_k, num_splits), msg,
+                                               sizeof(msg));
+  if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
+  moa::t_last_error[0] = '\0';
+  return MOA_OK;
+}
+
 const char* moa_last_error(void) { return moa::t_last_error; }
 
 int moa_get_device_status(void* stream) {
