@@ -66,7 +66,9 @@ def _load(path: str | None = None):
                                               ctypes.c_double, f64p, ctypes.c_int]
         lib.moa_oracle_attn_shifted_f64.argtypes = [f32p, f32p, f32p, f64p, i64, i64, i64, i64,
                                                     i64, i64, ctypes.c_double, f64p, ctypes.c_int]
-        for name in ("moa_oracle_attn_f64", "moa_oracle_rows_f64", "moa_oracle_weights_f64",
+        lib.moa_oracle_attn_lse_f64.argtypes = [f32p, f32p, f32p, f64p, f64p, i64, i64, i64,
+                                                i64, i64, i64, ctypes.c_double, ctypes.c_int]
+        for name in ("moa_oracle_attn_lse_f64", "moa_oracle_attn_f64", "moa_oracle_rows_f64", "moa_oracle_weights_f64",
                      "moa_oracle_scores_f64", "moa_oracle_attn_shifted_f64",
                      "moa_oracle_max_threads"):
             getattr(lib, name).restype = ctypes.c_int
@@ -180,6 +182,22 @@ class Oracle:
                                                   int(nthreads))
         self._check(rc, "moa_oracle_attn_shifted_f64")
         return out[0, 0] if squeeze else out
+
+    def attn_lse(self, q, k, v, scale: float, nthreads: int = 0):
+        """(O, LSE): the output and, per output row, ln sum_k exp(scale * <q_i, k_k>)."""
+        squeeze = np.ndim(q) == 2
+        q, k, v, (B, H, Nq, Nk, dk, dv) = self._dims(q, k, v)
+        q, qp = self._f32(q)
+        k, kp = self._f32(k)
+        v, vp = self._f32(v)
+        out = np.empty((B, H, Nq, dv), dtype=np.float64)
+        lse = np.empty((B, H, Nq), dtype=np.float64)
+        dp = ctypes.POINTER(ctypes.c_double)
+        rc = self.lib.moa_oracle_attn_lse_f64(qp, kp, vp, out.ctypes.data_as(dp),
+                                              lse.ctypes.data_as(dp), B, H, Nq, Nk, dk, dv,
+                                              float(scale), int(nthreads))
+        self._check(rc, "moa_oracle_attn_lse_f64")
+        return (out[0, 0], lse[0, 0]) if squeeze else (out, lse)
 
     def max_threads(self) -> int:
         return int(self.lib.moa_oracle_max_threads())

@@ -77,7 +77,7 @@ static void row_scores(const oracle_problem *p, int64_t row, double *s)
  * output_dnf).  w_out, if not NULL, receives the weights; o_out, if not NULL,
  * receives the output row. */
 static void row_softmax_output(const oracle_problem *p, int64_t row, double *s, double *e,
-                               double *w, double *w_out, double *o_out)
+                               double *w, double *w_out, double *o_out, double *lse_out)
 {
     const int64_t bh = row / p->Nq;
     const float *Vh = p->V + bh * p->Nk * p->dv;
@@ -91,6 +91,8 @@ static void row_softmax_output(const oracle_problem *p, int64_t row, double *s, 
         Z += e[k];
     for (int64_t k = 0; k < p->Nk; ++k)
         w[k] = e[k] / Z;
+    /* log of the denominator of Eq. stable_softmax before the shift: ln sum_k exp(s[k]) */
+    if (lse_out) *lse_out = m + log(Z);
     if (w_out)
         for (int64_t k = 0; k < p->Nk; ++k)
             w_out[k] = w[k];
@@ -107,7 +109,8 @@ static void row_softmax_output(const oracle_problem *p, int64_t row, double *s, 
  * shift, if not NULL, adds shift[r] to every score of output row r before the
  * softmax (used only to test shift invariance). */
 static int run_rows(const oracle_problem *p, const int64_t *rows, int64_t nrows,
-                    const double *shift, double *W, double *S, double *O, int nthreads)
+                    const double *shift, double *W, double *S, double *O, double *LSE,
+                    int nthreads)
 {
     if (check_problem(p)) return -1;
     if (nrows < 0) return -1;
@@ -142,7 +145,7 @@ static int run_rows(const oracle_problem *p, const int64_t *rows, int64_t nrows,
                     for (int64_t k = 0; k < p->Nk; ++k)
                         S[r * p->Nk + k] = s[k];
                 row_softmax_output(p, row, s, e, w, W ? W + r * p->Nk : NULL,
-                                   O ? O + r * p->dv : NULL);
+                                   O ? O + r * p->dv : NULL, LSE ? LSE + r : NULL);
             }
             free(buf);
         }
@@ -157,7 +160,7 @@ int moa_oracle_attn_f64(const float *Q, const float *K, const float *V, double *
 {
     oracle_problem p = {Q, K, V, B, H, Nq, Nk, dk, dv, scale};
     if (!O) return -1;
-    return run_rows(&p, NULL, check_problem(&p) ? 0 : B * H * Nq, NULL, NULL, NULL, O, nthreads);
+    return run_rows(&p, NULL, check_problem(&p) ? 0 : B * H * Nq, NULL, NULL, NULL, O, NULL, nthreads);
 }
 
 /* Output rows for a list of flattened row indices r = (b*H + h)*Nq + i;
@@ -168,7 +171,7 @@ int moa_oracle_rows_f64(const float *Q, const float *K, const float *V, double *
 {
     oracle_problem p = {Q, K, V, B, H, Nq, Nk, dk, dv, scale};
     if (!O || !rows) return -1;
-    return run_rows(&p, rows, nrows, NULL, NULL, NULL, O, nthreads);
+    return run_rows(&p, rows, nrows, NULL, NULL, NULL, O, NULL, nthreads);
 }
 
 /* Attention weights W[B,H,Nq,Nk] (Eq. dnf_attn) and, if O is not NULL, the
@@ -179,7 +182,7 @@ int moa_oracle_weights_f64(const float *Q, const float *K, const float *V, doubl
 {
     oracle_problem p = {Q, K, V, B, H, Nq, Nk, dk, dv, scale};
     if (!W) return -1;
-    return run_rows(&p, NULL, check_problem(&p) ? 0 : B * H * Nq, NULL, W, NULL, O, nthreads);
+    return run_rows(&p, NULL, check_problem(&p) ? 0 : B * H * Nq, NULL, W, NULL, O, NULL, nthreads);
 }
 
 /* Scaled scores S[B,H,Nq,Nk] (Step 1 of Algorithm 1 only).  Meant for small
@@ -209,7 +212,19 @@ int moa_oracle_attn_shifted_f64(const float *Q, const float *K, const float *V, 
 {
     oracle_problem p = {Q, K, V, B, H, Nq, Nk, dk, dv, scale};
     if (!O || !shift) return -1;
-    return run_rows(&p, NULL, check_problem(&p) ? 0 : B * H * Nq, shift, NULL, NULL, O, nthreads);
+    return run_rows(&p, NULL, check_problem(&p) ? 0 : B * H * Nq, shift, NULL, NULL, O, NULL, nthreads);
+}
+
+/* Output O and, per output row, LSE = ln sum_k exp(s[k]) (the scaled scores' log-sum-exp,
+ * i.e. m + ln Z of Algorithm 1); LSE has B*H*Nq entries. */
+int moa_oracle_attn_lse_f64(const float *Q, const float *K, const float *V, double *O,
+                            double *LSE, int64_t B, int64_t H, int64_t Nq, int64_t Nk,
+                            int64_t dk, int64_t dv, double scale, int nthreads)
+{
+    oracle_problem p = {Q, K, V, B, H, Nq, Nk, dk, dv, scale};
+    if (!O || !LSE) return -1;
+    return run_rows(&p, NULL, check_problem(&p) ? 0 : B * H * Nq, NULL, NULL, NULL, O, LSE,
+                    nthreads);
 }
 
 /* Threads an OpenMP region would use by default (1 without OpenMP). */

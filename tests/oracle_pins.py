@@ -267,6 +267,40 @@ def pin_rows_and_threads(o):
     assert np.array_equal(got, full1.reshape(-1, 8)[rows])
 
 
+def pin_lse(o):
+    """Log-sum-exp of the scaled scores: decimal brute force, one key, and shift behaviour."""
+    ctx = decimal.Context(prec=50)
+    r = _rng(311)
+    Q = _f32(r.normal(size=(4, 5)) * 3)
+    K = _f32(r.normal(size=(6, 5)))
+    V = _f32(r.normal(size=(6, 2)))
+    _, lse = o.attn_lse(Q, K, V, 0.6)
+    for i in range(4):
+        tot = decimal.Decimal(0)
+        for kk in range(6):
+            s = decimal.Decimal(0)
+            for j in range(5):
+                s = ctx.add(s, ctx.multiply(decimal.Decimal(float(Q[i, j])), decimal.Decimal(float(K[kk, j]))))
+            tot = ctx.add(tot, ctx.exp(ctx.multiply(s, decimal.Decimal(0.6))))
+        assert abs(lse[i] - float(ctx.ln(tot))) <= 1e-13 * max(1.0, abs(lse[i]))
+    # one key: lse = its scaled score; V plays no part
+    K1 = K[:1]
+    _, l1 = o.attn_lse(Q, K1, V[:1], 0.6)
+    assert np.max(np.abs(l1 - 0.6 * (Q.astype(np.float64) @ K1[0].astype(np.float64)))) <= 1e-12
+    _, l2 = o.attn_lse(Q, K, V * 3 + 1, 0.6)
+    assert np.array_equal(lse, l2)
+    # K[..,0] = 1, Q[..,0] = delta: every score of row i moves by scale*delta, lse too
+    Ka = K.copy()
+    Ka[:, 0] = 1.0
+    Qa = Q.copy()
+    Qa[:, 0] = 0.0
+    Qb = Qa.copy()
+    Qb[:, 0] = _f32([1.0, -2.0, 4.0, 8.0])
+    _, la = o.attn_lse(Qa, Ka, V, 0.5)
+    _, lb = o.attn_lse(Qb, Ka, V, 0.5)
+    assert np.max(np.abs((lb - la) - 0.5 * np.array([1.0, -2.0, 4.0, 8.0]))) <= 1e-12
+
+
 ALL_PINS = [
     pin_paper_example,
     pin_decimal_bruteforce,
@@ -282,4 +316,5 @@ ALL_PINS = [
     pin_large_scores_stable,
     pin_planted_rows,
     pin_rows_and_threads,
+    pin_lse,
 ]

@@ -31,6 +31,8 @@ MUTANTS = {
                           "const float *Kh = p->K;"),
     "wrong_query_row": ("const float *q = p->Q + (bh * p->Nq + i) * p->dk;",
                         "const float *q = p->Q + (bh * p->Nq) * p->dk;"),
+    "lse_without_max": ("if (lse_out) *lse_out = m + log(Z);", "if (lse_out) *lse_out = log(Z);"),
+    "lse_log2": ("if (lse_out) *lse_out = m + log(Z);", "if (lse_out) *lse_out = m + log2(Z);"),
 }
 
 
