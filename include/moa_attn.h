@@ -80,6 +80,27 @@ int moa_attn_fwd(const void* Q, const void* K, const void* V, void* O, int64_t B
                  void* stream);
 
 /*
+ * moa_attn_fwd_lse -- moa_attn_fwd, and also the log-sum-exp of every row's scores.
+ *
+ * Defines: O as in moa_attn_fwd, plus, for every b, h, i,
+ *     LSE[b,h,i] = ln sum_{k < N_k} exp(s_k) = m + ln sum_k exp(s_k - m),  m = max_k s_k,
+ * i.e. the logarithm of the softmax denominator of Eq. (stable_softmax) before its
+ * max shift.  It is the per-row quantity a backward pass needs to rebuild the
+ * weights exp(s_k - LSE) without the N_q x N_k matrix (paper Stage 5, Section 9),
+ * and the one a merge of key ranges computed apart needs.
+ *
+ * Arguments: those of moa_attn_fwd, plus
+ *   LSE  device pointer, float32 [B, H, N_q] contiguous, natural logarithm; written,
+ *        4-byte aligned, must not overlap Q, K, V or O.  Owned by the caller.
+ * Accuracy: bf16 path, the kernel's exp2/log2 in fp32 of the fp32-accumulated
+ * scores (absolute error about 1e-5 * |LSE| + 1e-5); fp32 path, fp32 expf/logf.
+ * Behaviour: as moa_attn_fwd; LSE adds 4 bytes per output row of traffic.
+ */
+int moa_attn_fwd_lse(const void* Q, const void* K, const void* V, void* O, float* LSE, int64_t B,
+                     int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v, float scale,
+                     int dtype, void* stream);
+
+/*
  * moa_attn_fwd_staged -- the same computation with host-resident inputs and output.
  *
  * Defines: as moa_attn_fwd (paper Section 4.1, Eq. attention).  Copies hQ, hK,

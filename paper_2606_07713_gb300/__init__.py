@@ -16,13 +16,14 @@ import math
 from ._lib import (MOA_BF16, MOA_FP32, MoaError, check, lib, moa_attn_dnf_bytes,  # noqa: F401
                    moa_attn_flops, moa_attn_fwd, moa_attn_fwd_staged, moa_attn_version,
                    moa_get_device_status, moa_last_error, moa_selftest_wait_timeout,
-                   moa_attn_fwd_splitkv, moa_attn_splitkv_workspace_bytes)
+                   moa_attn_fwd_splitkv, moa_attn_splitkv_workspace_bytes, moa_attn_fwd_lse)
 
 __all__ = ["attn_fwd", "attn_fwd_staged", "get_device_status", "attn_flops", "dnf_bytes",
            "MOA_FP32", "MOA_BF16", "MoaError", "moa_attn_fwd", "moa_attn_fwd_staged",
            "moa_last_error", "moa_get_device_status", "moa_attn_flops", "moa_attn_dnf_bytes",
            "moa_attn_version", "moa_selftest_wait_timeout", "attn_fwd_splitkv",
-           "moa_attn_fwd_splitkv", "moa_attn_splitkv_workspace_bytes"]
+           "moa_attn_fwd_splitkv", "moa_attn_splitkv_workspace_bytes", "attn_fwd_lse",
+           "moa_attn_fwd_lse"]
 
 
 def _dtype_code(t) -> int:
@@ -72,6 +73,35 @@ def attn_fwd(q, k, v, scale: float | None = None, out=None, stream=None):
         check(moa_attn_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), B, H, Nq, Nk,
                            dk, dv, float(scale), code, s.cuda_stream))
     return out
+
+
+def attn_fwd_lse(q, k, v, scale: float | None = None, out=None, lse=None, stream=None):
+    """(O, LSE): attn_fwd's output and the float32 [B, H, N_q] natural-log log-sum-exp of each
+    row's scaled scores, ln sum_k exp(scale <q_i, k_k>)."""
+    import torch
+    for t in (q, k, v):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError("attn_fwd_lse needs contiguous CUDA tensors")
+    if not (q.dtype == k.dtype == v.dtype):
+        raise TypeError("q, k, v must share one dtype")
+    code = _dtype_code(q)
+    B, H, Nq, Nk, dk, dv = _dims(q, k, v)
+    if scale is None:
+        scale = 1.0 / math.sqrt(dk)
+    if out is None:
+        out = torch.empty((B, H, Nq, dv), dtype=q.dtype, device=q.device)
+    elif out.shape != (B, H, Nq, dv) or out.dtype != q.dtype or not out.is_contiguous():
+        raise ValueError("out has the wrong shape, dtype or layout")
+    if lse is None:
+        lse = torch.empty((B, H, Nq), dtype=torch.float32, device=q.device)
+    elif lse.shape != (B, H, Nq) or lse.dtype != torch.float32 or not lse.is_contiguous():
+        raise ValueError("lse must be a contiguous float32 [B, H, N_q] tensor")
+    with torch.cuda.device(q.device):
+        s = stream if stream is not None else torch.cuda.current_stream(q.device)
+        check(moa_attn_fwd_lse(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                               lse.data_ptr(), B, H, Nq, Nk, dk, dv, float(scale), code,
+                               s.cuda_stream))
+    return out, lse
 
 
 def attn_fwd_splitkv(q, k, v, num_splits: int, scale: float | None = None, out=None,

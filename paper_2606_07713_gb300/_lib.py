@@ -37,6 +37,8 @@ _I64 = ctypes.c_int64
 SIGNATURES = {
     "moa_attn_fwd": (ctypes.c_int, [_VP, _VP, _VP, _VP, _I64, _I64, _I64, _I64, _I64, _I64,
                                     ctypes.c_float, ctypes.c_int, _VP]),
+    "moa_attn_fwd_lse": (ctypes.c_int, [_VP, _VP, _VP, _VP, _VP, _I64, _I64, _I64, _I64, _I64,
+                                        _I64, ctypes.c_float, ctypes.c_int, _VP]),
     "moa_attn_fwd_staged": (ctypes.c_int, [_VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _I64, _I64,
                                            _I64, _I64, _I64, _I64, ctypes.c_float, ctypes.c_int,
                                            _VP]),
@@ -97,6 +99,10 @@ def check(status: int) -> None:
 # -- thin wrappers with the C names ----------------------------------------------------------
 def moa_attn_fwd(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream) -> int:
     return lib().moa_attn_fwd(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream)
+
+
+def moa_attn_fwd_lse(Q, K, V, O, LSE, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream) -> int:
+    return lib().moa_attn_fwd_lse(Q, K, V, O, LSE, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream)
 
 
 def moa_attn_fwd_staged(hQ, hK, hV, hO, dQ, dK, dV, dO, B, H, N_q, N_k, d_k, d_v, scale, dtype,

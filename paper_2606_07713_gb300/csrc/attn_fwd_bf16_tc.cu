@@ -163,6 +163,13 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
+// log2 by the MUFU lg2 instruction (absolute error about 2^-22 for the row sums l >= 1 used here).
+__device__ __forceinline__ float lg2_approx(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);  // .x (low 16 bits) = lo
   return *reinterpret_cast<uint32_t*>(&v);
@@ -249,7 +256,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmV, __nv_bfloat16* __restrict__ O,
                         int Nq, int Nk, int n_qblocks, float c_log2, uint64_t wait_limit_ns,
                         int n_splits, int kv_per_split, float* __restrict__ ws_o,
-                        float2* __restrict__ ws_ml) {
+                        float2* __restrict__ ws_ml, float* __restrict__ lse) {
   using C = Cfg<DK, DV>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -642,6 +649,11 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       tc_fence_before_sync();
       mbar_arrive(p_ready(j));
     }
+    // Natural-log LSE of the scaled scores, final once the loop is done: m and l are in log2
+    // units of c_log2 * s, and l is relative to m whether or not the last maximum update was
+    // taken (lazy rescale).
+    if (!SPLIT && lse != nullptr && ok && q0 + j * kBM + row < Nq)
+      lse[size_t(bh) * Nq + q0 + j * kBM + row] = (m + lg2_approx(l)) * 0.69314718055994531f;
     // Epilogue, Step IV: O / l -> bf16 -> global.  With a split key axis this CTA instead
     // writes its unnormalised fp32 O rows and (m, l) for the merge kernel.
     if (SPLIT && ok && wait_bounded(o_done(j), 0, wc)) {
@@ -802,6 +814,10 @@ template <int DK, int DV>
 int launch_tc(const AttnArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
               const CUtensorMap& mv, const SplitPlan& sp, void* ws, char* msg, size_t msglen) {
   using C = Cfg<DK, DV>;
+  if (sp.n_splits > 1 && a.lse != nullptr) {
+    snprintf(msg, msglen, "the log-sum-exp output is not available with a split key axis");
+    return 1;
+  }
   auto kern = sp.n_splits > 1 ? attn_fwd_bf16_tc_kernel<DK, DV, true>
                               : attn_fwd_bf16_tc_kernel<DK, DV, false>;
   static std::once_flag once;
@@ -831,7 +847,7 @@ int launch_tc(const AttnArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
                       : nullptr;
   kern<<<dim3(unsigned(grid)), dim3(kThreads), C::kSmemBytes, a.stream>>>(
       mq, mk, mv, static_cast<__nv_bfloat16*>(a.O), int(a.Nq), int(a.Nk), int(n_qblocks), c_log2,
-      wait_limit_ns(), sp.n_splits, sp.kv_per_split, ws_o, ws_ml);
+      wait_limit_ns(), sp.n_splits, sp.kv_per_split, ws_o, ws_ml, a.lse);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     snprintf(msg, msglen, "bf16 kernel launch: %s", cudaGetErrorString(e));

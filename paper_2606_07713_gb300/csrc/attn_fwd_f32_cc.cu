@@ -41,8 +41,9 @@ struct F32Smem {
 
 __global__ void __launch_bounds__(kThreads)
 attn_fwd_f32_cc_kernel(const float* __restrict__ Q, const float* __restrict__ K,
-                       const float* __restrict__ V, float* __restrict__ O, int Nq, int Nk, int dk,
-                       int dv, int n_qtiles, float scale) {
+                       const float* __restrict__ V, float* __restrict__ O,
+                       float* __restrict__ lse, int Nq, int Nk, int dk, int dv, int n_qtiles,
+                       float scale) {
   extern __shared__ float smem[];
   float* sQ = smem;                          // [kBM][dk]
   float* sK = sQ + kBM * dk;                 // [kBN][dk+1]
@@ -156,6 +157,8 @@ attn_fwd_f32_cc_kernel(const float* __restrict__ Q, const float* __restrict__ K,
     const int row = q0 + warp * kRowsPerWarp + r;
     if (row >= Nq) continue;
     const float inv = 1.0f / l[r];
+    // ln sum_k exp(scale s_k) = m + ln l (m is the exact row maximum here).
+    if (lse != nullptr && lane == 0) lse[bh * Nq + row] = m[r] + logf(l[r]);
 #pragma unroll
     for (int g = 0; g < kMaxColGroups; ++g) {
       const int c = lane + 32 * g;
@@ -182,8 +185,8 @@ int launch_attn_fwd_f32(const AttnArgs& a, char* msg, size_t msglen) {
   }
   attn_fwd_f32_cc_kernel<<<dim3(unsigned(grid)), dim3(kThreads), smem, a.stream>>>(
       static_cast<const float*>(a.Q), static_cast<const float*>(a.K),
-      static_cast<const float*>(a.V), static_cast<float*>(a.O), int(a.Nq), int(a.Nk), int(a.dk),
-      int(a.dv), n_qtiles, a.scale);
+      static_cast<const float*>(a.V), static_cast<float*>(a.O), a.lse, int(a.Nq), int(a.Nk),
+      int(a.dk), int(a.dv), n_qtiles, a.scale);
   e = cudaGetLastError();
   if (e != cudaSuccess) {
     snprintf(msg, msglen, "fp32 kernel launch: %s", cudaGetErrorString(e));

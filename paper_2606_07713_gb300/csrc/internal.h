@@ -15,6 +15,8 @@ struct AttnArgs {
   int64_t B, H, Nq, Nk, dk, dv;
   float scale;
   cudaStream_t stream;
+  // Optional per-row log-sum-exp output, fp32 [B*H*N_q] (nullptr: not written).
+  float* lse = nullptr;
 };
 
 // How the key axis of the bf16 kernel is split: n_splits contiguous ranges of kv_per_split

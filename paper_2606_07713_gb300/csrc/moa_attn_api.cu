@@ -105,8 +105,8 @@ int validate(const void* Q, const void* K, const void* V, void* O, int64_t B, in
 
 int dispatch(const void* Q, const void* K, const void* V, void* O, int64_t B, int64_t H,
              int64_t Nq, int64_t Nk, int64_t dk, int64_t dv, float scale, int dtype,
-             void* stream) {
-  AttnArgs a{Q, K, V, O, B, H, Nq, Nk, dk, dv, scale, static_cast<cudaStream_t>(stream)};
+             void* stream, float* lse = nullptr) {
+  AttnArgs a{Q, K, V, O, B, H, Nq, Nk, dk, dv, scale, static_cast<cudaStream_t>(stream), lse};
   char msg[256] = {0};
   const int rc = dtype == MOA_BF16 ? launch_attn_fwd_bf16(a, msg, sizeof(msg))
                                    : launch_attn_fwd_f32(a, msg, sizeof(msg));
@@ -127,6 +127,23 @@ int moa_attn_fwd(const void* Q, const void* K, const void* V, void* O, int64_t B
   const int rc = moa::validate(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
   if (rc != MOA_OK) return rc;
   return moa::dispatch(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream);
+}
+
+int moa_attn_fwd_lse(const void* Q, const void* K, const void* V, void* O, float* LSE, int64_t B,
+                     int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v, float scale,
+                     int dtype, void* stream) {
+  int64_t sz[4];
+  const int rc = moa::validate(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
+  if (rc != MOA_OK) return rc;
+  if (LSE == nullptr) return moa::fail(MOA_ERR_INVALID_ARG, "null LSE pointer");
+  if (reinterpret_cast<uintptr_t>(LSE) % 4 != 0)
+    return moa::fail(MOA_ERR_MISALIGNED, "LSE pointer is not 4-byte aligned");
+  const int64_t lse_bytes = B * H * N_q * 4;  // validate() bounded B*H*N_q*d_q*4
+  const void* ins[4] = {Q, K, V, O};
+  for (int i = 0; i < 4; ++i)
+    if (moa::overlaps(LSE, lse_bytes, ins[i], sz[i]))
+      return moa::fail(MOA_ERR_INVALID_ARG, "LSE overlaps a tensor");
+  return moa::dispatch(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream, LSE);
 }
 
 int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO, void* dQ,

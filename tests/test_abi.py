@@ -110,3 +110,15 @@ def test_splitkv_validation_without_gpu(L):
     assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 4, None, 0, None) == _lib.MOA_ERR_INVALID_ARG
     assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 4, 0x500008, 1 << 20, None) == _lib.MOA_ERR_MISALIGNED
     assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 4, D, 1 << 20, None) == _lib.MOA_ERR_INVALID_ARG
+
+
+def test_lse_validation_without_gpu(L):
+    f = _lib.moa_attn_fwd_lse
+    E = 0x500000
+    ok_args = (1, 1, 8, 8, 64, 64, 0.125, 1, None)
+    assert f(A, B_, C, D, None, *ok_args) == _lib.MOA_ERR_INVALID_ARG        # no LSE buffer
+    assert f(A, B_, C, D, E + 2, *ok_args) == _lib.MOA_ERR_MISALIGNED        # not 4-byte aligned
+    assert f(A, B_, C, D, D + 4, *ok_args) == _lib.MOA_ERR_INVALID_ARG       # LSE inside O
+    assert f(A, B_, C, D, A, *ok_args) == _lib.MOA_ERR_INVALID_ARG           # LSE aliases Q
+    assert f(None, B_, C, D, E, *ok_args) == _lib.MOA_ERR_INVALID_ARG        # the usual checks too
+    assert f(A, B_, C, D, E, 1, 1, 8, 8, 96, 64, 0.125, 1, None) == _lib.MOA_ERR_UNSUPPORTED_SHAPE
