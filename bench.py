@@ -4,14 +4,19 @@ Default workload: bf16 SDPA forward, B=4, H=16, N_q=N_k=2048, d_k=d_v=64, Q/K/V 
 N(0,1) from the seeded generator, scale=1/sqrt(d_k), no mask.  One step = one attention
 forward over that batch (the whole hot path: one kernel launch).
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload ID]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference|classical]
+                    [--workload ID] [--shape B,H,N_q,N_k,d_k,d_v]
 
 Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s: FLOPs of every step on every
 rank divided by the slowest rank's summed kernel time, measured with CUDA events on the
 launching stream, with L2 flushed (a 256 MiB write) before every step.  `e2e` is the same
 metric through moa_attn_fwd_staged (host buffers in and out, copies inside the timed region).
 `--impl reference` times the fp64 CPU oracle on the host cores instead (a bounded sample of
-rows per step).  Multi-GPU (torchrun): every rank runs its own full copy of the workload (the
+rows per step).  `--impl classical` times the step-by-step path whose traffic the paper's
+M_classical models (Section 8.2): the score matrix, its max-shifted exponentials and the
+normalised weights each materialised in device memory by eager PyTorch ops (cuBLAS GEMMs and
+elementwise/reduction kernels) -- a measurement of the comparison, not part of the library.
+`--shape` replaces the workload's sizes (bf16, same generator) for traffic sweeps.  Multi-GPU (torchrun): every rank runs its own full copy of the workload (the
 (b, h) problems are independent; no collective on the data path), so scaling is weak.
 """
 from __future__ import annotations
@@ -299,6 +304,75 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
 
 
 # ------------------------------------------------------------------------------------------
+# the classical path (what Eq. M_classical counts), for the measured traffic comparison
+# ------------------------------------------------------------------------------------------
+def classical_step(q, k, v, scale):
+    """Eq. attention evaluated the classical way, every intermediate a device array: scaled
+    scores (N_q x N_k), their row maxima, the shifted exponentials (N_q x N_k), the row sums,
+    the normalised weights (N_q x N_k), then the product with V."""
+    import torch
+    scores = torch.matmul(q, k.transpose(-2, -1)) * scale
+    shifted = scores - scores.amax(dim=-1, keepdim=True)
+    expo = torch.exp(shifted)
+    den = expo.sum(dim=-1, keepdim=True)
+    weights = expo / den
+    return torch.matmul(weights, v)
+
+
+def analytic_traffic(s: I.AttnShape) -> dict:
+    """Eqs. M_classical and M_MoA in elements, for N_q x N_k scores (the paper writes n for both)."""
+    nn = s.N_q * s.N_k
+    m_cl = s.B * s.H * (3 * nn + s.N_q * s.d_k + s.N_k * s.d_k + s.N_q + s.N_k * s.d_v)
+    m_moa = s.B * s.H * (s.N_q * s.d_k + s.N_k * s.d_k + s.N_k * s.d_v)
+    return {"M_classical_elements": m_cl, "M_moa_elements": m_moa,
+            "k_analytic": round(m_cl / m_moa, 3)}
+
+
+def run_classical(args, cfg: I.AttnConfig) -> None:
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0 or cfg.dtype != "bf16":
+        if rank == 0:
+            print(json.dumps({"impl": "classical", "unavailable": "bf16 workloads only"}))
+        return
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    s = cfg.shape
+    x = I.make_inputs(cfg)
+    q, k, v = (to_device_bf16(b, dev) for b in (x.q_bits, x.k_bits, x.v_bits))
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(args.warmup):
+        o = classical_step(q, k, v, cfg.scale)
+    torch.cuda.synchronize(dev)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        o = classical_step(q, k, v, cfg.scale)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize(dev)
+    total_ms = float(np.sum([a.elapsed_time(b) for a, b in ev]))
+    flops = 2.0 * s.B * s.H * s.N_q * s.N_k * (s.d_k + s.d_v)
+    # the classical path computes the same function as the library (untimed check)
+    import paper_2606_07713_gb300 as pkg
+    ref = pkg.attn_fwd(q, k, v, cfg.scale).float()
+    err = float((o.float() - ref).abs().max() / ref.abs().max())
+    line = {
+        "impl": "classical", "metric": METRIC,
+        "value": round(flops * args.steps / (total_ms * 1e-3) / 1e12, 2), "unit": "TFLOP/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(total_ms / args.steps, 6), "higher_is_better": True,
+        "dtype": "bf16", "data": "synthetic: seeded splitmix64 + Box-Muller inputs",
+        "config": dict(workload_desc(cfg), l2="not flushed; the N_q x N_k arrays exceed L2"),
+        "analytic": analytic_traffic(s),
+        "dnf_bytes": 2.0 * s.B * s.H * (s.N_q * s.d_k + s.N_k * s.d_k + s.N_k * s.d_v + s.N_q * s.d_v),
+        "rel_err_vs_library": err,
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------------------
 # the oracle on the host cores (cpu_baseline leg and --impl reference)
 # ------------------------------------------------------------------------------------------
 def _oracle_rows(cfg, x, nrows, seed):
@@ -383,16 +457,25 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=20)
-    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--impl", choices=["ours", "reference", "classical"], default="ours")
     ap.add_argument("--workload", type=int, default=DEFAULT_WORKLOAD, choices=sorted(I.CONFIGS))
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle time for the cpu_baseline sample")
+    ap.add_argument("--shape", default=None,
+                    help="B,H,N_q,N_k,d_k,d_v: a bf16 workload of this shape instead of --workload")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     cfg = I.CONFIGS[args.workload]
+    if args.shape:
+        dims = [int(t) for t in args.shape.split(",")]
+        if len(dims) != 6 or min(dims) < 1:
+            ap.error("--shape needs six positive integers B,H,N_q,N_k,d_k,d_v")
+        cfg = I.custom_config(*dims, dtype="bf16", seed=sum(dims))
     if args.impl == "reference":
         run_reference(args, cfg)
+    elif args.impl == "classical":
+        run_classical(args, cfg)
     else:
         run_ours(args, cfg)
 
