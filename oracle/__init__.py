@@ -68,7 +68,10 @@ def _load(path: str | None = None):
                                                     i64, i64, ctypes.c_double, f64p, ctypes.c_int]
         lib.moa_oracle_attn_lse_f64.argtypes = [f32p, f32p, f32p, f64p, f64p, i64, i64, i64,
                                                 i64, i64, i64, ctypes.c_double, ctypes.c_int]
-        for name in ("moa_oracle_attn_lse_f64", "moa_oracle_attn_f64", "moa_oracle_rows_f64", "moa_oracle_weights_f64",
+        lib.moa_oracle_attn_bwd_f64.argtypes = [f32p, f32p, f32p, f32p, f64p, f64p, f64p, i64,
+                                                i64, i64, i64, i64, i64, ctypes.c_double,
+                                                ctypes.c_int]
+        for name in ("moa_oracle_attn_bwd_f64", "moa_oracle_attn_lse_f64", "moa_oracle_attn_f64", "moa_oracle_rows_f64", "moa_oracle_weights_f64",
                      "moa_oracle_scores_f64", "moa_oracle_attn_shifted_f64",
                      "moa_oracle_max_threads"):
             getattr(lib, name).restype = ctypes.c_int
@@ -198,6 +201,30 @@ class Oracle:
                                               float(scale), int(nthreads))
         self._check(rc, "moa_oracle_attn_lse_f64")
         return (out[0, 0], lse[0, 0]) if squeeze else (out, lse)
+
+    def attn_bwd(self, q, k, v, do, scale: float, nthreads: int = 0):
+        """(dQ, dK, dV) of L with dL/dO = do, for O = softmax(scale Q K^T) V, in fp64."""
+        squeeze = np.ndim(q) == 2
+        q, k, v, (B, H, Nq, Nk, dk, dv) = self._dims(q, k, v)
+        if squeeze:
+            do = np.asarray(do)[None, None]
+        if tuple(np.shape(do)) != (B, H, Nq, dv):
+            raise ValueError(f"dO must be {(B, H, Nq, dv)}, got {np.shape(do)}")
+        q, qp = self._f32(q)
+        k, kp = self._f32(k)
+        v, vp = self._f32(v)
+        g, gp = self._f32(do)
+        dq = np.empty((B, H, Nq, dk), dtype=np.float64)
+        dkk = np.empty((B, H, Nk, dk), dtype=np.float64)
+        dvv = np.empty((B, H, Nk, dv), dtype=np.float64)
+        dp = ctypes.POINTER(ctypes.c_double)
+        rc = self.lib.moa_oracle_attn_bwd_f64(qp, kp, vp, gp, dq.ctypes.data_as(dp),
+                                              dkk.ctypes.data_as(dp), dvv.ctypes.data_as(dp),
+                                              B, H, Nq, Nk, dk, dv, float(scale), int(nthreads))
+        self._check(rc, "moa_oracle_attn_bwd_f64")
+        if squeeze:
+            return dq[0, 0], dkk[0, 0], dvv[0, 0]
+        return dq, dkk, dvv
 
     def max_threads(self) -> int:
         return int(self.lib.moa_oracle_max_threads())

@@ -27,6 +27,9 @@
  * same on x86-64 and AArch64.  OpenMP splits the work over whole rows only, so
  * the result is bit-identical for any thread count.
  *
+ * moa_oracle_attn_lse_f64 also returns each row's log-sum-exp, and moa_oracle_attn_bwd_f64
+ * the gradients dQ, dK, dV of the backward pass (Stage 5, Section 9) for a given dL/dO.
+ *
  * Inputs are float32 arrays holding the stored values exactly (bf16 and fp32
  * values both embed exactly in float32); every element is widened to double
  * before use.  scale is taken as given (the paper fixes 1/sqrt(d_k)).
@@ -225,6 +228,94 @@ int moa_oracle_attn_lse_f64(const float *Q, const float *K, const float *V, doub
     if (!O || !LSE) return -1;
     return run_rows(&p, NULL, check_problem(&p) ? 0 : B * H * Nq, NULL, NULL, NULL, O, LSE,
                     nthreads);
+}
+
+/*
+ * Backward pass of Eq. attention (paper Stage 5, Section 9).  With L a scalar loss and
+ * dO = dL/dO given, the paper writes the query gradient as
+ *     dL/dQ = dL/dO . V^T . (d softmax / d scaled scores) . K * scale,
+ * where the softmax Jacobian of one row with weights w is J = diag(w) - w w^T (dense N_k x N_k).
+ * J is symmetric and is applied here without being formed: for dP = dO V^T (one row),
+ *     J dP = w * (dP - w.dP)      (elementwise; w.dP is one number per row).
+ * dK and dV follow from the same chain rule applied to the other two operands of Eq.
+ * attention (the paper derives only dQ; these are the standard derivatives of the same
+ * expression):
+ *     dS = J dP (per row),  dQ = scale * dS K,  dK = scale * dS^T Q,  dV = W^T dO.
+ * One (b,h) slice per thread; inside a slice the rows are taken in index order, so the
+ * dK and dV sums have a fixed order and the result does not depend on the thread count.
+ * dQ is [B,H,Nq,dk], dK [B,H,Nk,dk], dV [B,H,Nk,dv].
+ */
+int moa_oracle_attn_bwd_f64(const float *Q, const float *K, const float *V, const float *dO,
+                            double *dQ, double *dK, double *dV, int64_t B, int64_t H,
+                            int64_t Nq, int64_t Nk, int64_t dk, int64_t dv, double scale,
+                            int nthreads)
+{
+    oracle_problem p = {Q, K, V, B, H, Nq, Nk, dk, dv, scale};
+    if (!dO || !dQ || !dK || !dV || check_problem(&p)) return -1;
+    int status = 0;
+#ifdef _OPENMP
+    if (nthreads <= 0) nthreads = omp_get_max_threads();
+#pragma omp parallel num_threads(nthreads)
+#endif
+    {
+        double *buf = (double *)malloc(sizeof(double) * 5 * (size_t)Nk);
+        if (!buf) {
+#ifdef _OPENMP
+#pragma omp atomic write
+#endif
+            status = -2;
+        } else {
+            double *s = buf, *e = buf + Nk, *w = buf + 2 * Nk, *dP = buf + 3 * Nk;
+            double *dS = buf + 4 * Nk;
+#ifdef _OPENMP
+#pragma omp for schedule(dynamic, 1)
+#endif
+            for (int64_t bh = 0; bh < B * H; ++bh) {
+                const float *Kh = K + bh * Nk * dk;
+                const float *Vh = V + bh * Nk * dv;
+                double *dKh = dK + bh * Nk * dk;
+                double *dVh = dV + bh * Nk * dv;
+                for (int64_t t = 0; t < Nk * dk; ++t) dKh[t] = 0.0;
+                for (int64_t t = 0; t < Nk * dv; ++t) dVh[t] = 0.0;
+                for (int64_t i = 0; i < Nq; ++i) {
+                    const int64_t row = bh * Nq + i;
+                    const float *q = Q + row * dk;
+                    const float *g = dO + row * dv;
+                    /* forward weights of this row (Algorithm 1) */
+                    row_scores(&p, row, s);
+                    row_softmax_output(&p, row, s, e, w, NULL, NULL, NULL);
+                    /* dP = dO_i V^T, then the Jacobian product dS = w * (dP - w.dP) */
+                    for (int64_t k = 0; k < Nk; ++k) {
+                        double acc = 0.0;
+                        for (int64_t c = 0; c < dv; ++c)
+                            acc += (double)g[c] * (double)Vh[k * dv + c];
+                        dP[k] = acc;
+                    }
+                    double wdp = 0.0;
+                    for (int64_t k = 0; k < Nk; ++k)
+                        wdp += w[k] * dP[k];
+                    for (int64_t k = 0; k < Nk; ++k)
+                        dS[k] = w[k] * (dP[k] - wdp);
+                    /* dQ_i = scale * dS K */
+                    for (int64_t j = 0; j < dk; ++j) {
+                        double acc = 0.0;
+                        for (int64_t k = 0; k < Nk; ++k)
+                            acc += dS[k] * (double)Kh[k * dk + j];
+                        dQ[row * dk + j] = scale * acc;
+                    }
+                    /* dK_k += scale * dS_k q_i,  dV_k += w_k dO_i */
+                    for (int64_t k = 0; k < Nk; ++k) {
+                        for (int64_t j = 0; j < dk; ++j)
+                            dKh[k * dk + j] += scale * dS[k] * (double)q[j];
+                        for (int64_t c = 0; c < dv; ++c)
+                            dVh[k * dv + c] += w[k] * (double)g[c];
+                    }
+                }
+            }
+            free(buf);
+        }
+    }
+    return status;
 }
 
 /* Threads an OpenMP region would use by default (1 without OpenMP). */

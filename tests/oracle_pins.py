@@ -301,6 +301,111 @@ def pin_lse(o):
     assert np.max(np.abs((lb - la) - 0.5 * np.array([1.0, -2.0, 4.0, 8.0]))) <= 1e-12
 
 
+# ----------------------------------------------------------------------------------------------
+# 4. Backward pass (Stage 5): gradients of L = sum(dO * O)
+# ----------------------------------------------------------------------------------------------
+def _decimal_loss(Q, K, V, G, scale, ctx):
+    """L = sum_ic G[i,c] * O[i,c] with O = softmax(scale Q K^T) V, all in decimal arithmetic;
+    Q, K, V, G are nested lists of Decimals."""
+    nq, nk, dk, dv = len(Q), len(K), len(Q[0]), len(V[0])
+    total = decimal.Decimal(0)
+    for i in range(nq):
+        ex = []
+        for k in range(nk):
+            s = decimal.Decimal(0)
+            for j in range(dk):
+                s = ctx.add(s, ctx.multiply(Q[i][j], K[k][j]))
+            ex.append(ctx.exp(ctx.multiply(s, scale)))
+        z = decimal.Decimal(0)
+        for e in ex:
+            z = ctx.add(z, e)
+        for c in range(dv):
+            acc = decimal.Decimal(0)
+            for k in range(nk):
+                acc = ctx.add(acc, ctx.multiply(ex[k], V[k][c]))
+            total = ctx.add(total, ctx.multiply(G[i][c], ctx.divide(acc, z)))
+    return total
+
+
+def pin_bwd_finite_differences(o):
+    """Every gradient entry against a central difference of the loss in 60-digit decimal
+    arithmetic (step 1e-12: truncation ~1e-24, rounding ~1e-48)."""
+    ctx = decimal.Context(prec=60)
+    D = lambda x: decimal.Decimal(float(x))
+    for t, (nq, nk, dk, dv, scale) in enumerate([(3, 4, 3, 2, 0.7), (2, 5, 2, 3, -1.3)]):
+        r = _rng(400 + t)
+        Q = _f32(r.normal(size=(nq, dk)) * 1.5)
+        K = _f32(r.normal(size=(nk, dk)))
+        V = _f32(r.normal(size=(nk, dv)))
+        G = _f32(r.normal(size=(nq, dv)))
+        dq, dkk, dvv = o.attn_bwd(Q, K, V, G, scale)
+        mats = [[[D(x) for x in row] for row in M] for M in (Q, K, V)]
+        g = [[D(x) for x in row] for row in G]
+        sc = D(scale)
+        h = decimal.Decimal("1e-12")
+        for which, grad in enumerate((dq, dkk, dvv)):
+            M = mats[which]
+            for a in range(len(M)):
+                for b in range(len(M[0])):
+                    keep = M[a][b]
+                    M[a][b] = keep + h
+                    lp = _decimal_loss(mats[0], mats[1], mats[2], g, sc, ctx)
+                    M[a][b] = keep - h
+                    lm = _decimal_loss(mats[0], mats[1], mats[2], g, sc, ctx)
+                    M[a][b] = keep
+                    fd = float(ctx.divide(ctx.subtract(lp, lm), 2 * h))
+                    assert abs(grad[a, b] - fd) <= 1e-12 * max(1.0, abs(fd)), (t, which, a, b)
+
+
+def pin_bwd_closed_forms(o):
+    """One key: dQ = dK = 0 and dV = sum_i dO_i.  scale = 0: dQ = dK = 0 and dV_k = mean
+    over keys of sum_i dO_i.  Identical value rows: dQ = dK = 0."""
+    r = _rng(410)
+    Q = _f32(r.normal(size=(2, 3, 7, 8)) * 3)
+    K = _f32(r.normal(size=(2, 3, 1, 8)))
+    V = _f32(r.normal(size=(2, 3, 1, 5)))
+    G = _f32(r.normal(size=(2, 3, 7, 5)))
+    dq, dkk, dvv = o.attn_bwd(Q, K, V, G, 0.8)
+    assert np.max(np.abs(dq)) == 0.0 and np.max(np.abs(dkk)) == 0.0
+    assert np.max(np.abs(dvv[:, :, 0] - G.astype(np.float64).sum(axis=2))) <= 1e-13
+    K = _f32(r.normal(size=(2, 3, 9, 8)))
+    V = _f32(r.normal(size=(2, 3, 9, 5)))
+    dq, dkk, dvv = o.attn_bwd(Q, K, V, G, 0.0)
+    assert np.max(np.abs(dq)) == 0.0 and np.max(np.abs(dkk)) == 0.0
+    mean = G.astype(np.float64).sum(axis=2, keepdims=True) / 9.0
+    assert np.max(np.abs(dvv - mean)) <= 1e-13
+    Vs = np.broadcast_to(V[:, :, :1], V.shape).copy()
+    dq, dkk, _ = o.attn_bwd(Q, K, Vs, G, 0.5)
+    assert np.max(np.abs(dq)) <= 1e-13 and np.max(np.abs(dkk)) <= 1e-13
+
+
+def pin_bwd_invariants(o):
+    """Each row of dS sums to zero, so the dK rows of a head sum to zero; the weights of a row
+    sum to one, so the dV rows of a head sum to sum_i dO_i; by homogeneity of the scores in
+    Q and in K, <dQ, Q> = <dK, K> per head; and the gradients are linear in dO."""
+    r = _rng(411)
+    Q = _f32(r.normal(size=(2, 2, 13, 16)) * 2)
+    K = _f32(r.normal(size=(2, 2, 21, 16)))
+    V = _f32(r.normal(size=(2, 2, 21, 6)))
+    # dO values on a 1/64 grid, so that G1 + G2 is exact in float32
+    G1 = _f32(np.round(r.normal(size=(2, 2, 13, 6)) * 64) / 64)
+    G2 = _f32(np.round(r.normal(size=(2, 2, 13, 6)) * 64) / 64)
+    dq, dkk, dvv = o.attn_bwd(Q, K, V, G1, 0.3)
+    assert np.max(np.abs(dkk.sum(axis=2))) <= 1e-12 * np.max(np.abs(dkk))
+    assert np.max(np.abs(dvv.sum(axis=2) - G1.astype(np.float64).sum(axis=2))) <= 1e-12
+    qq = np.einsum("bhij,bhij->bh", dq, Q.astype(np.float64))
+    kk = np.einsum("bhkj,bhkj->bh", dkk, K.astype(np.float64))
+    assert np.max(np.abs(qq - kk)) <= 1e-12 * np.max(np.abs(qq))
+    a = o.attn_bwd(Q, K, V, G1, 0.3)
+    b = o.attn_bwd(Q, K, V, G2, 0.3)
+    c = o.attn_bwd(Q, K, V, G1.astype(np.float64) + G2.astype(np.float64), 0.3)
+    for x, y, z in zip(a, b, c):
+        assert np.max(np.abs(x + y - z)) <= 1e-12 * max(1.0, np.max(np.abs(z)))
+    # thread count does not change any bit
+    assert all(np.array_equal(x, y) for x, y in zip(o.attn_bwd(Q, K, V, G1, 0.3, nthreads=1),
+                                                    o.attn_bwd(Q, K, V, G1, 0.3, nthreads=3)))
+
+
 ALL_PINS = [
     pin_paper_example,
     pin_decimal_bruteforce,
@@ -317,4 +422,7 @@ ALL_PINS = [
     pin_planted_rows,
     pin_rows_and_threads,
     pin_lse,
+    pin_bwd_finite_differences,
+    pin_bwd_closed_forms,
+    pin_bwd_invariants,
 ]

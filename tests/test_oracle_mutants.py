@@ -33,6 +33,16 @@ MUTANTS = {
                         "const float *q = p->Q + (bh * p->Nq) * p->dk;"),
     "lse_without_max": ("if (lse_out) *lse_out = m + log(Z);", "if (lse_out) *lse_out = log(Z);"),
     "lse_log2": ("if (lse_out) *lse_out = m + log(Z);", "if (lse_out) *lse_out = m + log2(Z);"),
+    "bwd_drops_rank_one_term": ("dS[k] = w[k] * (dP[k] - wdp);", "dS[k] = w[k] * dP[k];"),
+    "bwd_sign_flipped": ("dS[k] = w[k] * (dP[k] - wdp);", "dS[k] = w[k] * (wdp - dP[k]);"),
+    "bwd_dk_without_scale": ("dKh[k * dk + j] += scale * dS[k] * (double)q[j];",
+                             "dKh[k * dk + j] += dS[k] * (double)q[j];"),
+    "bwd_dv_from_ds": ("dVh[k * dv + c] += w[k] * (double)g[c];",
+                       "dVh[k * dv + c] += dS[k] * (double)g[c];"),
+    "bwd_dp_v_transposed": ("acc += (double)g[c] * (double)Vh[k * dv + c];",
+                            "acc += (double)g[c] * (double)Vh[c * Nk + k];"),
+    "bwd_dq_uses_q": ("acc += dS[k] * (double)Kh[k * dk + j];",
+                      "acc += dS[k] * (double)Kh[j];"),
 }
 
 
