@@ -101,6 +101,51 @@ int moa_attn_fwd_lse(const void* Q, const void* K, const void* V, void* O, float
                      int dtype, void* stream);
 
 /*
+ * moa_attn_bwd -- gradients of a scalar loss through O = softmax(scale * Q K^T) V.
+ *
+ * Defines: paper Stage 5 (Section 9) gives the query gradient as
+ *     dL/dQ = dL/dO . V^T . J . K * scale,  J the row-wise Jacobian of the softmax;
+ * with W the attention weights and dP = dO V^T, J applied to a row of dP is
+ * w * (dP - w.dP), so for every (b, h):
+ *     dS = W * (dO V^T - D),  D_i = sum_c dO[i,c] O[i,c]  (= w_i . dP_i),
+ *     dQ = scale * dS K,  dK = scale * dS^T Q,  dV = W^T dO.
+ * (dK and dV are the derivatives of the same expression with respect to its other two
+ * operands.)  W is rebuilt from the scores and LSE; no N_q x N_k array is written to
+ * device memory.
+ *
+ * Arguments:
+ *   Q, K, V  device, the forward inputs (layouts of moa_attn_fwd), read only
+ *   O        device, [B, H, N_q, d_v], the forward output for these inputs, read only
+ *   dO       device, [B, H, N_q, d_v], dL/dO, read only
+ *   LSE      device, float32 [B, H, N_q], the forward pass's log-sum-exp (moa_attn_fwd_lse)
+ *   dQ, dK, dV  device, written: [B, H, N_q, d_k], [B, H, N_k, d_k], [B, H, N_k, d_v]
+ *   B, H, N_q, N_k, d_k, d_v, scale   as for moa_attn_fwd (the same scale as the forward)
+ *   dtype    MOA_BF16 only (MOA_ERR_UNSUPPORTED_DTYPE otherwise); gradients are bf16
+ *   workspace, workspace_bytes  device scratch of at least moa_attn_bwd_workspace_bytes(...)
+ *            bytes, 16-byte aligned, owned by the caller; its contents need no initial value
+ *   stream   a cudaStream_t of the current device
+ * Supported sizes: d_k, d_v in {64, 128}; the limits of moa_attn_fwd.  Alignment: every
+ * tensor 16-byte aligned (LSE 4-byte).  Outputs and workspace must not overlap each other
+ * or any input.
+ * Behaviour: asynchronous; three kernel launches on `stream` (per-row D and LSE in log2
+ * units, then dK/dV, then dQ).  Allocates nothing.  Bounded waits as for moa_attn_fwd
+ * (moa_get_device_status reports a timeout).  Accumulation is fp32 in tensor memory; the
+ * weights W and dS enter the tensor-core products rounded to bf16.
+ */
+int moa_attn_bwd(const void* Q, const void* K, const void* V, const void* O, const void* dO,
+                 const float* LSE, void* dQ, void* dK, void* dV, int64_t B, int64_t H,
+                 int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v, float scale, int dtype,
+                 void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * moa_attn_bwd_workspace_bytes -- scratch bytes moa_attn_bwd needs: two fp32 values per
+ * (b, h) and query row, rows padded to a multiple of 128 (0 for a dtype without a backward
+ * or sizes < 1).
+ */
+size_t moa_attn_bwd_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int64_t d_k,
+                                    int64_t d_v, int dtype);
+
+/*
  * moa_attn_fwd_staged -- the same computation with host-resident inputs and output.
  *
  * Defines: as moa_attn_fwd (paper Section 4.1, Eq. attention).  Copies hQ, hK,

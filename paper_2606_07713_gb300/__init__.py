@@ -16,14 +16,15 @@ import math
 from ._lib import (MOA_BF16, MOA_FP32, MoaError, check, lib, moa_attn_dnf_bytes,  # noqa: F401
                    moa_attn_flops, moa_attn_fwd, moa_attn_fwd_staged, moa_attn_version,
                    moa_get_device_status, moa_last_error, moa_selftest_wait_timeout,
-                   moa_attn_fwd_splitkv, moa_attn_splitkv_workspace_bytes, moa_attn_fwd_lse)
+                   moa_attn_fwd_splitkv, moa_attn_splitkv_workspace_bytes, moa_attn_fwd_lse,
+                   moa_attn_bwd, moa_attn_bwd_workspace_bytes)
 
 __all__ = ["attn_fwd", "attn_fwd_staged", "get_device_status", "attn_flops", "dnf_bytes",
            "MOA_FP32", "MOA_BF16", "MoaError", "moa_attn_fwd", "moa_attn_fwd_staged",
            "moa_last_error", "moa_get_device_status", "moa_attn_flops", "moa_attn_dnf_bytes",
            "moa_attn_version", "moa_selftest_wait_timeout", "attn_fwd_splitkv",
            "moa_attn_fwd_splitkv", "moa_attn_splitkv_workspace_bytes", "attn_fwd_lse",
-           "moa_attn_fwd_lse"]
+           "moa_attn_fwd_lse", "attn_bwd", "moa_attn_bwd", "moa_attn_bwd_workspace_bytes"]
 
 
 def _dtype_code(t) -> int:
@@ -102,6 +103,38 @@ def attn_fwd_lse(q, k, v, scale: float | None = None, out=None, lse=None, stream
                                lse.data_ptr(), B, H, Nq, Nk, dk, dv, float(scale), code,
                                s.cuda_stream))
     return out, lse
+
+
+def attn_bwd(q, k, v, o, lse, do, scale: float | None = None, workspace=None, stream=None):
+    """(dQ, dK, dV) for O = softmax(scale q k^T) v given dO = dL/dO, from the forward's o and lse
+    (attn_fwd_lse).  bf16 CUDA tensors [B, H, N, d]; lse float32 [B, H, N_q]."""
+    import torch
+    for t in (q, k, v, o, do, lse):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError("attn_bwd needs contiguous CUDA tensors")
+    if not (q.dtype == k.dtype == v.dtype == o.dtype == do.dtype):
+        raise TypeError("q, k, v, o, do must share one dtype")
+    code = _dtype_code(q)
+    B, H, Nq, Nk, dk, dv = _dims(q, k, v)
+    if tuple(o.shape) != (B, H, Nq, dv) or tuple(do.shape) != (B, H, Nq, dv):
+        raise ValueError("o and do must be [B, H, N_q, d_v]")
+    if tuple(lse.shape) != (B, H, Nq) or lse.dtype != torch.float32:
+        raise ValueError("lse must be float32 [B, H, N_q]")
+    if scale is None:
+        scale = 1.0 / math.sqrt(dk)
+    dq = torch.empty_like(q)
+    dkk = torch.empty_like(k)
+    dvv = torch.empty_like(v)
+    need = moa_attn_bwd_workspace_bytes(B, H, Nq, Nk, dk, dv, code)
+    if workspace is None:
+        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=q.device)
+    with torch.cuda.device(q.device):
+        s = stream if stream is not None else torch.cuda.current_stream(q.device)
+        check(moa_attn_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(), do.data_ptr(),
+                           lse.data_ptr(), dq.data_ptr(), dkk.data_ptr(), dvv.data_ptr(), B, H, Nq,
+                           Nk, dk, dv, float(scale), code, workspace.data_ptr(), workspace.numel(),
+                           s.cuda_stream))
+    return dq, dkk, dvv
 
 
 def attn_fwd_splitkv(q, k, v, num_splits: int, scale: float | None = None, out=None,

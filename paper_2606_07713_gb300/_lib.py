@@ -39,6 +39,11 @@ SIGNATURES = {
                                     ctypes.c_float, ctypes.c_int, _VP]),
     "moa_attn_fwd_lse": (ctypes.c_int, [_VP, _VP, _VP, _VP, _VP, _I64, _I64, _I64, _I64, _I64,
                                         _I64, ctypes.c_float, ctypes.c_int, _VP]),
+    "moa_attn_bwd": (ctypes.c_int, [_VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _I64, _I64, _I64,
+                                    _I64, _I64, _I64, ctypes.c_float, ctypes.c_int, _VP,
+                                    ctypes.c_size_t, _VP]),
+    "moa_attn_bwd_workspace_bytes": (ctypes.c_size_t, [_I64, _I64, _I64, _I64, _I64, _I64,
+                                                       ctypes.c_int]),
     "moa_attn_fwd_staged": (ctypes.c_int, [_VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _I64, _I64,
                                            _I64, _I64, _I64, _I64, ctypes.c_float, ctypes.c_int,
                                            _VP]),
@@ -103,6 +108,16 @@ def moa_attn_fwd(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream) -> 
 
 def moa_attn_fwd_lse(Q, K, V, O, LSE, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream) -> int:
     return lib().moa_attn_fwd_lse(Q, K, V, O, LSE, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream)
+
+
+def moa_attn_bwd(Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v, scale, dtype,
+                 workspace, workspace_bytes, stream) -> int:
+    return lib().moa_attn_bwd(Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v, scale,
+                              dtype, workspace, workspace_bytes, stream)
+
+
+def moa_attn_bwd_workspace_bytes(B, H, N_q, N_k, d_k, d_v, dtype) -> int:
+    return lib().moa_attn_bwd_workspace_bytes(B, H, N_q, N_k, d_k, d_v, dtype)
 
 
 def moa_attn_fwd_staged(hQ, hK, hV, hO, dQ, dK, dV, dO, B, H, N_q, N_k, d_k, d_v, scale, dtype,

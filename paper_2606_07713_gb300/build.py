@@ -1,6 +1,6 @@
 """Builds libmoa_attn.so from csrc/ with nvcc for sm_103a (in-tree, under _build/).
 
-The three translation units compile in parallel; the library links the CUDA
+The translation units compile in parallel; the library links the CUDA
 runtime statically and loads the driver's tensor-map encoder at run time, so it
 has no link-time dependency on libcuda and loads on machines without a GPU.
 """
@@ -16,8 +16,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libmoa_attn.so")
-SOURCES = ["moa_attn_api.cu", "attn_fwd_f32_cc.cu", "attn_fwd_bf16_tc.cu"]
-HEADERS = ["internal.h", "ptx.cuh"]
+SOURCES = ["moa_attn_api.cu", "attn_fwd_f32_cc.cu", "attn_fwd_bf16_tc.cu", "attn_bwd_bf16_tc.cu"]
+HEADERS = ["internal.h", "ptx.cuh", "tc_common.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xptxas", "-v"]
 

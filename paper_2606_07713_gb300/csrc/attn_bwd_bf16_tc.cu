@@ -1,0 +1,753 @@
+// bf16 attention backward on the fifth-generation tensor cores (tcgen05 + TMEM + TMA), sm_103a.
+//
+// What it computes (paper Stage 5, Section 9): for O = softmax(scale * Q K^T) V and a given
+// dO = dL/dO, the gradients
+//     dV = W^T dO,   dS = W * (dO V^T - D),   dQ = scale * dS K,   dK = scale * dS^T Q,
+// with W the attention weights and D_i = sum_c dO_ic O_ic = sum_k W_ik (dO V^T)_ik, which is
+// the softmax Jacobian (diag(w) - w w^T) applied row by row without ever forming it.  As in the
+// forward pass, no N_q x N_k array (scores, weights, dP, dS) exists in global memory: the
+// weights are rebuilt tile by tile from the scores and the forward pass's per-row log-sum-exp,
+// W_ik = exp2(c * s_ik - LSE_i * log2 e), c = scale * log2 e.
+//
+// Three kernels:
+//   attn_bwd_pre_kernel   per query row: D_i and -LSE_i * log2 e into a padded fp32 workspace
+//                         (rows past N_q get D = 0 and -inf, so padded queries weigh nothing);
+//   attn_bwd_dkdv_kernel  one CTA per (b, h, block of 128 keys); streams every 128-row query
+//                         block through a shared-memory ring and accumulates dV and dK in TMEM:
+//                           S^T = K Q^T, dP^T = V dO^T            (TMEM, fp32)
+//                           P^T = exp2(c S^T - L), dS^T = P^T (dP^T - D)   (registers, per key row)
+//                           dV += P^T dO,  dK += dS^T Q           (A operand from TMEM, bf16)
+//   attn_bwd_dq_kernel    one CTA per (b, h, block of 128 query rows); streams the key blocks:
+//                           S = Q K^T, dP = dO V^T, dS = P (dP - D), dQ += dS K.
+// Splitting dQ from dK/dV keeps every accumulation inside one CTA (no atomics, deterministic
+// results) at the price of computing S and dP twice: 7 tile products per (query, key) block
+// pair instead of 5.
+//
+// CTA organisation of both tile kernels (one CTA per SM: 512 TMEM columns):
+//   warps 0-7: 128 rows x 2 column halves.  Warp w owns TMEM lanes 32*(w%4).. (its rows) and
+//              columns [64*(w/4), +64) of the 128-wide score tiles; it writes its bf16 P or dS
+//              back into the first 32 of those columns, so the two halves never overlap.  The
+//              products that read them take K-steps 0-3 from columns 0-31 and 4-7 from 64-95.
+//   warp 8:    TMEM allocation and the single thread that issues every tcgen05.mma;
+//   warp 9:    the single thread that issues every TMA copy.
+// Every mbarrier wait is bounded; on expiry the kernel records MOA_ERR_DEVICE_TIMEOUT in
+// g_moa_bwd_status, every role leaves its loop, and TMEM is still freed.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdio>
+#include <mutex>
+
+#include "internal.h"
+#include "ptx.cuh"
+#include "tc_common.cuh"
+
+namespace moa {
+
+__device__ unsigned int g_moa_bwd_status = 0;
+
+namespace {
+
+using namespace ptx;
+using namespace tc;
+
+constexpr int kBlk = 128;          // rows of every tile (= TMEM lanes) and keys per key block
+constexpr int kThreads = 320;      // 8 compute warps, MMA warp, TMA warp
+constexpr int kMmaWarp = 8;        // also allocates and frees TMEM
+constexpr int kLoadWarp = 9;
+constexpr int kTmemCols = 512;
+constexpr int kPanelBytes = 128 * 128;  // one 128-byte-swizzle panel: 64 bf16 columns x 128 rows
+constexpr int kVecBytes = kBlk * 4;     // 128 fp32 per-row values
+constexpr float kLog2e = 1.4426950408889634f;
+
+__host__ __device__ constexpr int ring_stages(int dk, int dv) {
+  return dk + dv <= 128 ? 4 : (dk + dv <= 192 ? 3 : 2);
+}
+
+// TMEM column of K-step kk (16 rows of the reduction axis) of a bf16 operand written by the two
+// column halves: steps 0-3 from columns 0-31, steps 4-7 from columns 64-95.
+__device__ __forceinline__ uint32_t half_split_col(int kk) {
+  return kk < 4 ? uint32_t(kk * 8) : uint32_t(64 + (kk - 4) * 8);
+}
+
+// Loads 64 fp32 TMEM columns of this thread's lane (two x32 loads) and waits.
+__device__ __forceinline__ void tmem_load_row64(uint32_t taddr, uint32_t* r) {
+  tmem_ld_32x32b_x32(taddr, r);
+  tmem_ld_32x32b_x32(taddr + 32, r + 32);
+  tmem_wait_ld();
+  reg_anchor_x32(r);
+  reg_anchor_x32(r + 32);
+}
+
+// Writes ncols fp32 TMEM columns of this thread's lane, times mul, as bf16 to dst (16-B aligned).
+template <int NCOLS>
+__device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_bfloat16* dst,
+                                               bool valid) {
+#pragma unroll
+  for (int c = 0; c < NCOLS; c += 32) {
+    uint32_t o[32];
+    tmem_ld_32x32b_x32(taddr + c, o);
+    tmem_wait_ld();
+    reg_anchor_x32(o);
+    if (valid) {
+      uint4 pkt[4];
+      uint32_t* w = reinterpret_cast<uint32_t*>(pkt);
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        w[i] = pack_bf16x2(__uint_as_float(o[2 * i]) * mul, __uint_as_float(o[2 * i + 1]) * mul);
+      uint4* d4 = reinterpret_cast<uint4*>(dst + c);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) d4[i] = pkt[i];
+    }
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// Per-row preprocessing
+// ------------------------------------------------------------------------------------------
+// One warp per padded query row r = bh * Nq_pad + i:
+//   Dd[r] = sum_c dO[bh,i,c] * O[bh,i,c] (fp32 products of the bf16 values),
+//   nL[r] = -LSE[bh,i] * log2 e;  rows i >= N_q: Dd = 0, nL = -inf.
+template <int DV>
+__global__ void __launch_bounds__(256)
+attn_bwd_pre_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfloat16* __restrict__ dO,
+                    const float* __restrict__ lse, float* __restrict__ nL, float* __restrict__ Dd,
+                    int Nq, int Nq_pad, long long rows_pad) {
+  const long long r = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows_pad) return;
+  const long long bh = r / Nq_pad;
+  const int i = int(r % Nq_pad);
+  if (i >= Nq) {
+    if (lane == 0) {
+      nL[r] = -INFINITY;
+      Dd[r] = 0.f;
+    }
+    return;
+  }
+  const long long src = bh * Nq + i;
+  float acc = 0.f;
+  constexpr int kPer = DV / 32;  // bf16 elements per lane: 2 or 4
+  const __nv_bfloat16* o = O + src * DV + lane * kPer;
+  const __nv_bfloat16* g = dO + src * DV + lane * kPer;
+#pragma unroll
+  for (int t = 0; t < kPer; t += 2) {
+    const __nv_bfloat162 ov = *reinterpret_cast<const __nv_bfloat162*>(o + t);
+    const __nv_bfloat162 gv = *reinterpret_cast<const __nv_bfloat162*>(g + t);
+    const float2 of = __bfloat1622float2(ov), gf = __bfloat1622float2(gv);
+    acc = fmaf(of.x, gf.x, acc);
+    acc = fmaf(of.y, gf.y, acc);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  if (lane == 0) {
+    nL[r] = -lse[src] * kLog2e;
+    Dd[r] = acc;
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// dK and dV: one CTA per (b, h, 128-key block)
+// ------------------------------------------------------------------------------------------
+template <int DK, int DV>
+struct DkDvCfg {
+  static_assert((DK == 64 || DK == 128) && (DV == 64 || DV == 128), "d_k, d_v in {64, 128}");
+  static constexpr int kKBytes = kBlk * DK * 2;
+  static constexpr int kVBytes = kBlk * DV * 2;
+  static constexpr int kQBytes = kBlk * DK * 2;
+  static constexpr int kDOBytes = kBlk * DV * 2;
+  // stage: Q tile, dO tile, -L (log2 units) and D of its 128 rows; a multiple of 1024 bytes
+  static constexpr int kStageBytes = kQBytes + kDOBytes + 2 * kVecBytes;
+  static constexpr int kStages = ring_stages(DK, DV);
+  static constexpr int kOffK = 0;
+  static constexpr int kOffV = kKBytes;
+  static constexpr int kOffStage = kKBytes + kVBytes;
+  // barriers: full[NS], empty[NS], kv_full, s_full, dp_full, p_ready, ds_ready, acc_done
+  static constexpr int kNumBars = 2 * kStages + 6;
+  static constexpr int kOffBar = kOffStage + kStages * kStageBytes;
+  static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+  static constexpr int kSmemBytes = kOffMisc + 16 + 1024;
+  static constexpr uint32_t kTmemS = 0, kTmemDP = 128, kTmemDV = 256, kTmemDK = 256 + DV;
+  static_assert(kStageBytes % 1024 == 0, "stage alignment");
+  static_assert(kTmemDK + DK <= kTmemCols, "TMEM budget");
+  static_assert(kSmemBytes <= 232448, "shared memory budget");
+};
+
+template <int DK, int DV>
+__global__ void __launch_bounds__(kThreads, 1)
+attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                     const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmDO,
+                     const float* __restrict__ nL, const float* __restrict__ Dd,
+                     __nv_bfloat16* __restrict__ dK, __nv_bfloat16* __restrict__ dV, int Nk,
+                     int Nq_pad, int n_kblocks, float c_log2, float scale, uint64_t wait_limit_ns) {
+  using C = DkDvCfg<DK, DV>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  const uint32_t sK = smem_u32(smem + C::kOffK);
+  const uint32_t sV = smem_u32(smem + C::kOffV);
+  const uint32_t sStage = smem_u32(smem + C::kOffStage);
+  const uint32_t bar0 = smem_u32(smem + C::kOffBar);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (C::kStages + s); };
+  const uint32_t kv_full = bar0 + 8u * (2 * C::kStages);
+  const uint32_t s_full = kv_full + 8, dp_full = kv_full + 16, p_ready = kv_full + 24;
+  const uint32_t ds_ready = kv_full + 32, acc_done = kv_full + 40;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int bh = blockIdx.x / n_kblocks;
+  const int k0 = (blockIdx.x % n_kblocks) * kBlk;
+  const int n_qb = Nq_pad / kBlk;
+  const WaitCtl wc{abort_flag, wait_limit_ns, 0u, &g_moa_bwd_status};
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    mbar_init(kv_full, 1);
+    mbar_init(s_full, 1);
+    mbar_init(dp_full, 1);
+    mbar_init(p_ready, 8 * 32);
+    mbar_init(ds_ready, 8 * 32);
+    mbar_init(acc_done, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == kLoadWarp) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmQ);
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      tma_prefetch_desc(&tmDO);
+      mbar_arrive_expect_tx(kv_full, C::kKBytes + C::kVBytes);
+#pragma unroll
+      for (int p = 0; p < DK / 64; ++p)
+        tma_load_3d(sK + p * kPanelBytes, &tmK, kv_full, p * 64, k0, bh);
+#pragma unroll
+      for (int p = 0; p < DV / 64; ++p)
+        tma_load_3d(sV + p * kPanelBytes, &tmV, kv_full, p * 64, k0, bh);
+      int slot = 0;
+      uint32_t phase = 0, issued = 0, issued_phase = 0;
+      bool aborted = false;
+      for (int i = 0; i < n_qb; ++i) {
+        if (!wait_bounded(empty_bar(slot), phase ^ 1u, wc)) {
+          aborted = true;
+          break;
+        }
+        issued |= 1u << slot;
+        issued_phase = (issued_phase & ~(1u << slot)) | (phase << slot);
+        const uint32_t st = sStage + slot * C::kStageBytes;
+        mbar_arrive_expect_tx(full_bar(slot), C::kStageBytes);
+#pragma unroll
+        for (int p = 0; p < DK / 64; ++p)
+          tma_load_3d(st + p * kPanelBytes, &tmQ, full_bar(slot), p * 64, i * kBlk, bh);
+#pragma unroll
+        for (int p = 0; p < DV / 64; ++p)
+          tma_load_3d(st + C::kQBytes + p * kPanelBytes, &tmDO, full_bar(slot), p * 64, i * kBlk,
+                      bh);
+        const size_t vrow = size_t(bh) * Nq_pad + size_t(i) * kBlk;
+        bulk_load(st + C::kQBytes + C::kDOBytes, nL + vrow, kVecBytes, full_bar(slot));
+        bulk_load(st + C::kQBytes + C::kDOBytes + kVecBytes, Dd + vrow, kVecBytes, full_bar(slot));
+        if (++slot == C::kStages) {
+          slot = 0;
+          phase ^= 1u;
+        }
+      }
+      if (aborted || *abort_flag) {
+        wait_quiesce(kv_full, 0, wait_limit_ns, &g_moa_bwd_status);
+        for (int sl = 0; sl < C::kStages; ++sl)
+          if (issued & (1u << sl))
+            wait_quiesce(full_bar(sl), (issued_phase >> sl) & 1u, wait_limit_ns, &g_moa_bwd_status);
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t kIdescS = make_idesc(kBlk, kBlk, false);
+      constexpr uint32_t kIdescDV = make_idesc(kBlk, DV, true);
+      constexpr uint32_t kIdescDK = make_idesc(kBlk, DK, true);
+      const uint32_t tS = tmem + C::kTmemS, tDP = tmem + C::kTmemDP;
+      const uint32_t tDV = tmem + C::kTmemDV, tDK = tmem + C::kTmemDK;
+      int slot = 0;
+      uint32_t phase = 0;
+      bool ok = wait_bounded(kv_full, 0, wc);
+      for (int i = 0; ok && i < n_qb; ++i) {
+        const int st = slot;
+        ok = wait_bounded(full_bar(slot), phase, wc);
+        if (++slot == C::kStages) {
+          slot = 0;
+          phase ^= 1u;
+        }
+        if (!ok) break;
+        tc_fence_after_sync();
+        const uint32_t sQ = sStage + st * C::kStageBytes, sDO = sQ + C::kQBytes;
+        const uint32_t par = uint32_t(i) & 1u;
+        // S^T = K Q^T: M = 128 keys, N = 128 queries, both operands K-major (d_k contiguous);
+        // reduction step kk is panel kk/4, 32 bytes further per step inside it.
+#pragma unroll
+        for (int kk = 0; kk < DK / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
+          mma_f16_ss(tS, make_sdesc_sw128(sK + off, 16, 1024), make_sdesc_sw128(sQ + off, 16, 1024),
+                     kIdescS, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(s_full);
+        // dP^T = V dO^T: M = 128 keys, N = 128 queries, reduction over d_v.
+#pragma unroll
+        for (int kk = 0; kk < DV / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
+          mma_f16_ss(tDP, make_sdesc_sw128(sV + off, 16, 1024), make_sdesc_sw128(sDO + off, 16, 1024),
+                     kIdescS, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(dp_full);
+        // dV += P^T dO: A = P^T (bf16, TMEM), B = dO tile MN-major (d_v contiguous): groups of 8
+        // query rows 1024 B apart, 64-column panels kPanelBytes apart.
+        ok = wait_bounded(p_ready, par, wc);
+        if (!ok) break;
+        tc_fence_after_sync();
+#pragma unroll
+        for (int kk = 0; kk < kBlk / 16; ++kk)
+          mma_f16_ts(tDV, tS + half_split_col(kk),
+                     make_sdesc_sw128(sDO + kk * 2048, kPanelBytes, 1024), kIdescDV,
+                     (kk > 0 || i > 0) ? 1u : 0u);
+        // dK += dS^T Q (scale applied in the epilogue): B = Q tile MN-major.
+        ok = wait_bounded(ds_ready, par, wc);
+        if (!ok) break;
+        tc_fence_after_sync();
+#pragma unroll
+        for (int kk = 0; kk < kBlk / 16; ++kk)
+          mma_f16_ts(tDK, tDP + half_split_col(kk),
+                     make_sdesc_sw128(sQ + kk * 2048, kPanelBytes, 1024), kIdescDK,
+                     (kk > 0 || i > 0) ? 1u : 0u);
+        mma_commit(empty_bar(st));
+      }
+      // Always signal once everything issued has completed, so that TMEM is quiescent before
+      // it is freed even on the abort path.
+      mma_commit(acc_done);
+    }
+  } else {
+    // ---------------------------------------------------------------- compute warps
+    const int half = warp >> 2;              // column half of the 128-query tiles
+    const int lane_base = (warp & 3) * 32;   // TMEM lanes (key rows) of this warp
+    const int row = lane_base + lane;        // key row inside the block
+    const uint32_t lanes = uint32_t(lane_base) << 16;
+    const uint32_t tS = tmem + lanes + C::kTmemS + half * 64;
+    const uint32_t tDP = tmem + lanes + C::kTmemDP + half * 64;
+    const uint64_t cc = pack_f32x2(c_log2, c_log2);
+    int slot = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int i = 0; i < n_qb; ++i) {
+      const int st = slot;
+      const uint32_t par = uint32_t(i) & 1u;
+      // The stage's -L and D came with the tiles (TMA); waiting on its full barrier makes
+      // them visible to this thread.
+      ok = wait_bounded(full_bar(st), phase, wc) && wait_bounded(s_full, par, wc);
+      if (++slot == C::kStages) {
+        slot = 0;
+        phase ^= 1u;
+      }
+      if (!ok) break;
+      tc_fence_after_sync();
+      const float* vec = reinterpret_cast<const float*>(smem + C::kOffStage + st * C::kStageBytes +
+                                                        C::kQBytes + C::kDOBytes);
+      const float4* nl4 = reinterpret_cast<const float4*>(vec + half * 64);
+      const float4* d4 = reinterpret_cast<const float4*>(vec + kBlk + half * 64);
+      uint32_t r[64];
+      tmem_load_row64(tS, r);
+      float p[64];
+#pragma unroll
+      for (int q = 0; q < 64; q += 4) {
+        const float4 l = nl4[q >> 2];
+        ffma2(p[q], p[q + 1], __uint_as_float(r[q]), __uint_as_float(r[q + 1]), cc,
+              pack_f32x2(l.x, l.y));
+        ffma2(p[q + 2], p[q + 3], __uint_as_float(r[q + 2]), __uint_as_float(r[q + 3]), cc,
+              pack_f32x2(l.z, l.w));
+      }
+      uint32_t pk[32];
+#pragma unroll
+      for (int q = 0; q < 64; q += 2) {
+        p[q] = ex2_approx(p[q]);
+        p[q + 1] = ex2_approx(p[q + 1]);
+        pk[q >> 1] = pack_bf16x2(p[q], p[q + 1]);
+      }
+      tmem_st_32x32b_x32(tS, pk);
+      tmem_wait_st();
+      tc_fence_before_sync();
+      mbar_arrive(p_ready);
+      ok = wait_bounded(dp_full, par, wc);
+      if (!ok) break;
+      tc_fence_after_sync();
+      tmem_load_row64(tDP, r);
+#pragma unroll
+      for (int q = 0; q < 64; q += 4) {
+        const float4 d = d4[q >> 2];
+        const float s0 = p[q] * (__uint_as_float(r[q]) - d.x);
+        const float s1 = p[q + 1] * (__uint_as_float(r[q + 1]) - d.y);
+        const float s2 = p[q + 2] * (__uint_as_float(r[q + 2]) - d.z);
+        const float s3 = p[q + 3] * (__uint_as_float(r[q + 3]) - d.w);
+        pk[q >> 1] = pack_bf16x2(s0, s1);
+        pk[(q >> 1) + 1] = pack_bf16x2(s2, s3);
+      }
+      tmem_st_32x32b_x32(tDP, pk);
+      tmem_wait_st();
+      tc_fence_before_sync();
+      mbar_arrive(ds_ready);
+    }
+    // Epilogue: half 0 writes dV, half 1 writes scale * dK (rows past N_k are not stored).
+    if (ok && wait_bounded(acc_done, 0, wc)) {
+      tc_fence_after_sync();
+      const bool valid = k0 + row < Nk;
+      const size_t grow = size_t(bh) * Nk + size_t(k0 + row);
+      if (half == 0)
+        store_row_bf16<DV>(tmem + lanes + C::kTmemDV, 1.0f, dV + grow * DV, valid);
+      else
+        store_row_bf16<DK>(tmem + lanes + C::kTmemDK, scale, dK + grow * DK, valid);
+    }
+  }
+
+  if (warp == kMmaWarp) wait_quiesce(acc_done, 0, wait_limit_ns, &g_moa_bwd_status);
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after_sync();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// dQ: one CTA per (b, h, 128-row query block)
+// ------------------------------------------------------------------------------------------
+template <int DK, int DV>
+struct DqCfg {
+  static_assert((DK == 64 || DK == 128) && (DV == 64 || DV == 128), "d_k, d_v in {64, 128}");
+  static constexpr int kQBytes = kBlk * DK * 2;
+  static constexpr int kDOBytes = kBlk * DV * 2;
+  static constexpr int kKBytes = kBlk * DK * 2;
+  static constexpr int kVBytes = kBlk * DV * 2;
+  static constexpr int kStageBytes = kKBytes + kVBytes;  // K tile, V tile
+  static constexpr int kStages = ring_stages(DK, DV);
+  static constexpr int kOffQ = 0;
+  static constexpr int kOffDO = kQBytes;
+  static constexpr int kOffStage = kQBytes + kDOBytes;
+  // barriers: full[NS], empty[NS], q_full, s_full, dp_full, ds_ready, acc_done
+  static constexpr int kNumBars = 2 * kStages + 5;
+  static constexpr int kOffBar = kOffStage + kStages * kStageBytes;
+  static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+  static constexpr int kSmemBytes = kOffMisc + 16 + 1024;
+  static constexpr uint32_t kTmemS = 0, kTmemDP = 128, kTmemDQ = 256;
+  static_assert(kTmemDQ + DK <= kTmemCols, "TMEM budget");
+  static_assert(kSmemBytes <= 232448, "shared memory budget");
+};
+
+template <int DK, int DV>
+__global__ void __launch_bounds__(kThreads, 1)
+attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmDO,
+                   const float* __restrict__ nL, const float* __restrict__ Dd,
+                   __nv_bfloat16* __restrict__ dQ, int Nq, int Nk, int Nq_pad, int n_qblocks,
+                   float c_log2, float scale, uint64_t wait_limit_ns) {
+  using C = DqCfg<DK, DV>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  const uint32_t sQ = smem_u32(smem + C::kOffQ);
+  const uint32_t sDO = smem_u32(smem + C::kOffDO);
+  const uint32_t sStage = smem_u32(smem + C::kOffStage);
+  const uint32_t bar0 = smem_u32(smem + C::kOffBar);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (C::kStages + s); };
+  const uint32_t q_full = bar0 + 8u * (2 * C::kStages);
+  const uint32_t s_full = q_full + 8, dp_full = q_full + 16, ds_ready = q_full + 24;
+  const uint32_t acc_done = q_full + 32;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int bh = blockIdx.x / n_qblocks;
+  const int q0 = (blockIdx.x % n_qblocks) * kBlk;
+  const int n_kb = (Nk + kBlk - 1) / kBlk;
+  const WaitCtl wc{abort_flag, wait_limit_ns, 0u, &g_moa_bwd_status};
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    mbar_init(q_full, 1);
+    mbar_init(s_full, 1);
+    mbar_init(dp_full, 1);
+    mbar_init(ds_ready, 8 * 32);
+    mbar_init(acc_done, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == kLoadWarp) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmQ);
+      tma_prefetch_desc(&tmK);
+      tma_prefetch_desc(&tmV);
+      tma_prefetch_desc(&tmDO);
+      mbar_arrive_expect_tx(q_full, C::kQBytes + C::kDOBytes);
+#pragma unroll
+      for (int p = 0; p < DK / 64; ++p)
+        tma_load_3d(sQ + p * kPanelBytes, &tmQ, q_full, p * 64, q0, bh);
+#pragma unroll
+      for (int p = 0; p < DV / 64; ++p)
+        tma_load_3d(sDO + p * kPanelBytes, &tmDO, q_full, p * 64, q0, bh);
+      int slot = 0;
+      uint32_t phase = 0, issued = 0, issued_phase = 0;
+      bool aborted = false;
+      for (int j = 0; j < n_kb; ++j) {
+        if (!wait_bounded(empty_bar(slot), phase ^ 1u, wc)) {
+          aborted = true;
+          break;
+        }
+        issued |= 1u << slot;
+        issued_phase = (issued_phase & ~(1u << slot)) | (phase << slot);
+        const uint32_t st = sStage + slot * C::kStageBytes;
+        mbar_arrive_expect_tx(full_bar(slot), C::kStageBytes);
+#pragma unroll
+        for (int p = 0; p < DK / 64; ++p)
+          tma_load_3d(st + p * kPanelBytes, &tmK, full_bar(slot), p * 64, j * kBlk, bh);
+#pragma unroll
+        for (int p = 0; p < DV / 64; ++p)
+          tma_load_3d(st + C::kKBytes + p * kPanelBytes, &tmV, full_bar(slot), p * 64, j * kBlk,
+                      bh);
+        if (++slot == C::kStages) {
+          slot = 0;
+          phase ^= 1u;
+        }
+      }
+      if (aborted || *abort_flag) {
+        wait_quiesce(q_full, 0, wait_limit_ns, &g_moa_bwd_status);
+        for (int sl = 0; sl < C::kStages; ++sl)
+          if (issued & (1u << sl))
+            wait_quiesce(full_bar(sl), (issued_phase >> sl) & 1u, wait_limit_ns, &g_moa_bwd_status);
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t kIdescS = make_idesc(kBlk, kBlk, false);
+      constexpr uint32_t kIdescDQ = make_idesc(kBlk, DK, true);
+      const uint32_t tS = tmem + C::kTmemS, tDP = tmem + C::kTmemDP, tDQ = tmem + C::kTmemDQ;
+      int slot = 0;
+      uint32_t phase = 0;
+      bool ok = wait_bounded(q_full, 0, wc);
+      for (int j = 0; ok && j < n_kb; ++j) {
+        const int st = slot;
+        ok = wait_bounded(full_bar(slot), phase, wc);
+        if (++slot == C::kStages) {
+          slot = 0;
+          phase ^= 1u;
+        }
+        if (!ok) break;
+        tc_fence_after_sync();
+        const uint32_t sK = sStage + st * C::kStageBytes, sV = sK + C::kKBytes;
+        // S = Q K^T (M = 128 queries, N = 128 keys, K-major operands)
+#pragma unroll
+        for (int kk = 0; kk < DK / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
+          mma_f16_ss(tS, make_sdesc_sw128(sQ + off, 16, 1024), make_sdesc_sw128(sK + off, 16, 1024),
+                     kIdescS, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(s_full);
+        // dP = dO V^T (reduction over d_v)
+#pragma unroll
+        for (int kk = 0; kk < DV / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
+          mma_f16_ss(tDP, make_sdesc_sw128(sDO + off, 16, 1024), make_sdesc_sw128(sV + off, 16, 1024),
+                     kIdescS, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(dp_full);
+        // dQ += dS K (scale applied in the epilogue): A = dS (bf16, TMEM), B = K tile MN-major.
+        ok = wait_bounded(ds_ready, uint32_t(j) & 1u, wc);
+        if (!ok) break;
+        tc_fence_after_sync();
+#pragma unroll
+        for (int kk = 0; kk < kBlk / 16; ++kk)
+          mma_f16_ts(tDQ, tDP + half_split_col(kk),
+                     make_sdesc_sw128(sK + kk * 2048, kPanelBytes, 1024), kIdescDQ,
+                     (kk > 0 || j > 0) ? 1u : 0u);
+        mma_commit(empty_bar(st));
+      }
+      mma_commit(acc_done);
+    }
+  } else {
+    // ---------------------------------------------------------------- compute warps
+    const int half = warp >> 2;              // column half of the 128-key tiles
+    const int lane_base = (warp & 3) * 32;   // TMEM lanes (query rows) of this warp
+    const int row = lane_base + lane;
+    const uint32_t lanes = uint32_t(lane_base) << 16;
+    const uint32_t tS = tmem + lanes + C::kTmemS + half * 64;
+    const uint32_t tDP = tmem + lanes + C::kTmemDP + half * 64;
+    const size_t vrow = size_t(bh) * Nq_pad + size_t(q0 + row);  // padded: always in range
+    const float nl = nL[vrow], dd = Dd[vrow];
+    const uint64_t cc = pack_f32x2(c_log2, c_log2);
+    const uint64_t nn = pack_f32x2(nl, nl);
+    bool ok = true;
+    for (int j = 0; j < n_kb; ++j) {
+      const uint32_t par = uint32_t(j) & 1u;
+      ok = wait_bounded(s_full, par, wc);
+      if (!ok) break;
+      tc_fence_after_sync();
+      uint32_t r[64];
+      tmem_load_row64(tS, r);
+      float p[64];
+#pragma unroll
+      for (int k = 0; k < 64; k += 2) {
+        ffma2(p[k], p[k + 1], __uint_as_float(r[k]), __uint_as_float(r[k + 1]), cc, nn);
+        p[k] = ex2_approx(p[k]);
+        p[k + 1] = ex2_approx(p[k + 1]);
+      }
+      ok = wait_bounded(dp_full, par, wc);
+      if (!ok) break;
+      tc_fence_after_sync();
+      tmem_load_row64(tDP, r);
+      uint32_t pk[32];
+#pragma unroll
+      for (int k = 0; k < 64; k += 2)
+        pk[k >> 1] = pack_bf16x2(p[k] * (__uint_as_float(r[k]) - dd),
+                                 p[k + 1] * (__uint_as_float(r[k + 1]) - dd));
+      tmem_st_32x32b_x32(tDP, pk);
+      tmem_wait_st();
+      tc_fence_before_sync();
+      mbar_arrive(ds_ready);
+    }
+    // Epilogue: scale * dQ -> bf16; half h writes columns [h*DK/2, (h+1)*DK/2).
+    if (ok && wait_bounded(acc_done, 0, wc)) {
+      tc_fence_after_sync();
+      const bool valid = q0 + row < Nq;
+      __nv_bfloat16* dst = dQ + (size_t(bh) * Nq + size_t(valid ? q0 + row : 0)) * DK + half * (DK / 2);
+      store_row_bf16<DK / 2>(tmem + lanes + C::kTmemDQ + half * (DK / 2), scale, dst, valid);
+    }
+  }
+
+  if (warp == kMmaWarp) wait_quiesce(acc_done, 0, wait_limit_ns, &g_moa_bwd_status);
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after_sync();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------------------------------
+// Host side
+// ------------------------------------------------------------------------------------------
+int64_t padded_rows(int64_t Nq) { return (Nq + kBlk - 1) / kBlk * kBlk; }
+
+template <int DK, int DV>
+int launch_bwd(const BwdArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
+               const CUtensorMap& mv, const CUtensorMap& mdo, char* msg, size_t msglen) {
+  using A = DkDvCfg<DK, DV>;
+  using B = DqCfg<DK, DV>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [&] {
+    attr_err = cudaFuncSetAttribute(attn_bwd_dkdv_kernel<DK, DV>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, A::kSmemBytes);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(attn_bwd_dq_kernel<DK, DV>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, B::kSmemBytes);
+  });
+  if (attr_err != cudaSuccess) {
+    snprintf(msg, msglen, "cudaFuncSetAttribute (bf16 backward): %s", cudaGetErrorString(attr_err));
+    return 5;
+  }
+  const int64_t BH = a.B * a.H;
+  const int64_t nq_pad = padded_rows(a.Nq);
+  const int64_t n_kb = (a.Nk + kBlk - 1) / kBlk, n_qb = nq_pad / kBlk;
+  if (BH * n_kb > 0x7fffffffLL || BH * n_qb > 0x7fffffffLL || BH * nq_pad / 8 > 0x7fffffffLL ||
+      nq_pad > 0x7fffffffLL) {
+    snprintf(msg, msglen, "bf16 backward: grid too large");
+    return 3;
+  }
+  float* nL = static_cast<float*>(a.ws);
+  float* Dd = nL + BH * nq_pad;
+  const float c_log2 = a.scale * kLog2e;
+  const long long rows_pad = BH * nq_pad;
+  attn_bwd_pre_kernel<DV><<<dim3(unsigned((rows_pad + 7) / 8)), dim3(256), 0, a.stream>>>(
+      static_cast<const __nv_bfloat16*>(a.O), static_cast<const __nv_bfloat16*>(a.dO), a.lse, nL,
+      Dd, int(a.Nq), int(nq_pad), rows_pad);
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) {
+    attn_bwd_dkdv_kernel<DK, DV><<<dim3(unsigned(BH * n_kb)), dim3(kThreads), A::kSmemBytes,
+                                   a.stream>>>(
+        mq, mk, mv, mdo, nL, Dd, static_cast<__nv_bfloat16*>(a.dK),
+        static_cast<__nv_bfloat16*>(a.dV), int(a.Nk), int(nq_pad), int(n_kb), c_log2, a.scale,
+        wait_limit_ns());
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) {
+    attn_bwd_dq_kernel<DK, DV><<<dim3(unsigned(BH * n_qb)), dim3(kThreads), B::kSmemBytes,
+                                 a.stream>>>(mq, mk, mv, mdo, nL, Dd,
+                                             static_cast<__nv_bfloat16*>(a.dQ), int(a.Nq),
+                                             int(a.Nk), int(nq_pad), int(n_qb), c_log2, a.scale,
+                                             wait_limit_ns());
+    e = cudaGetLastError();
+  }
+  if (e != cudaSuccess) {
+    snprintf(msg, msglen, "bf16 backward launch: %s", cudaGetErrorString(e));
+    return 5;
+  }
+  return 0;
+}
+
+}  // namespace
+
+size_t bwd_workspace_bytes(int64_t B, int64_t H, int64_t Nq) {
+  return size_t(2) * size_t(B) * size_t(H) * size_t(padded_rows(Nq)) * sizeof(float);
+}
+
+int launch_attn_bwd_bf16(const BwdArgs& a, char* msg, size_t msglen) {
+  const int64_t BH = a.B * a.H;
+  CUtensorMap mq, mk, mv, mdo;
+  if (!encode_bf16_map(&mq, a.Q, BH, a.Nq, a.dk, msg, msglen)) return 5;
+  if (!encode_bf16_map(&mk, a.K, BH, a.Nk, a.dk, msg, msglen)) return 5;
+  if (!encode_bf16_map(&mv, a.V, BH, a.Nk, a.dv, msg, msglen)) return 5;
+  if (!encode_bf16_map(&mdo, a.dO, BH, a.Nq, a.dv, msg, msglen)) return 5;
+  if (a.dk == 64 && a.dv == 64) return launch_bwd<64, 64>(a, mq, mk, mv, mdo, msg, msglen);
+  if (a.dk == 128 && a.dv == 128) return launch_bwd<128, 128>(a, mq, mk, mv, mdo, msg, msglen);
+  if (a.dk == 128 && a.dv == 64) return launch_bwd<128, 64>(a, mq, mk, mv, mdo, msg, msglen);
+  if (a.dk == 64 && a.dv == 128) return launch_bwd<64, 128>(a, mq, mk, mv, mdo, msg, msglen);
+  snprintf(msg, msglen, "bf16 backward supports d_k, d_v in {64, 128}; got d_k=%lld d_v=%lld",
+           (long long)a.dk, (long long)a.dv);
+  return 3;
+}
+
+cudaError_t bwd_read_and_clear_status(unsigned* value) {
+  cudaError_t e = cudaMemcpyFromSymbol(value, g_moa_bwd_status, sizeof(unsigned));
+  if (e != cudaSuccess) return e;
+  const unsigned zero = 0;
+  return cudaMemcpyToSymbol(g_moa_bwd_status, &zero, sizeof(unsigned));
+}
+
+}  // namespace moa

@@ -49,6 +49,7 @@
 
 #include "internal.h"
 #include "ptx.cuh"
+#include "tc_common.cuh"
 
 namespace moa {
 
@@ -57,6 +58,7 @@ __device__ unsigned int g_moa_bf16_status = 0;
 namespace {
 
 using namespace ptx;
+using namespace tc;
 
 constexpr int kBM = 128;          // query rows per Q tile (= TMEM lanes)
 constexpr int kBN = 128;          // keys per K/V tile
@@ -105,102 +107,6 @@ struct Cfg {
   static_assert(kSmemBytes <= 232448, "shared memory budget");
 };
 
-// Instruction descriptor of tcgen05.mma kind::f16: D fp32, A and B bf16, dense.
-//   bits 4-5 D format (1 = f32), 7-9 A format (1 = bf16), 10-12 B format (1 = bf16),
-//   15 A major (0 = K-major), 16 B major (1 = MN-major), 17-22 N >> 3, 24-28 M >> 4.
-__host__ __device__ constexpr uint32_t make_idesc(int M, int N, bool b_mn_major) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | ((b_mn_major ? 1u : 0u) << 16) |
-         (uint32_t(N >> 3) << 17) | (uint32_t(M >> 4) << 24);
-}
-
-// Shared-memory matrix descriptor, 128-byte swizzle (layout code 2 in bits 61-63), version 1
-// (bits 46-47).  Start address, leading and stride byte offsets in 16-byte units.
-__device__ __forceinline__ uint64_t make_sdesc_sw128(uint32_t addr, uint32_t lbo, uint32_t sbo) {
-  return uint64_t((addr & 0x3FFFFu) >> 4) | (uint64_t((lbo >> 4) & 0x3FFFu) << 16) |
-         (uint64_t((sbo >> 4) & 0x3FFFu) << 32) | (uint64_t(1) << 46) | (uint64_t(2) << 61);
-}
-
-struct WaitCtl {
-  volatile int* abort_flag;
-  uint64_t limit_ns;
-  uint32_t hint_ns;  // 0: poll; otherwise let a not-yet-complete test suspend the thread
-};
-
-// Bounded mbarrier wait.  Returns false (and raises the CTA abort flag and the global status
-// word) if the phase did not complete within limit_ns, or if another role already aborted.
-__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, const WaitCtl& w) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer_ns();
-  for (uint32_t it = 1;; ++it) {
-    if (w.hint_ns ? mbar_try_wait_hint(bar, parity, w.hint_ns) : mbar_try_wait(bar, parity))
-      return true;
-    if ((it & 63u) == 0) {
-      if (*w.abort_flag) return false;
-      if (globaltimer_ns() - t0 > w.limit_ns) {
-        *w.abort_flag = 1;
-        atomicExch(&g_moa_bf16_status, 6u);  // MOA_ERR_DEVICE_TIMEOUT
-        return false;
-      }
-    }
-  }
-}
-
-// Time-limited wait that ignores the abort flag: used on the way out so that no TMA copy or
-// tensor-core operation is still writing shared or tensor memory when the CTA exits.
-__device__ __forceinline__ void wait_quiesce(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
-  const uint64_t t0 = globaltimer_ns();
-  while (!mbar_try_wait(bar, parity)) {
-    if (globaltimer_ns() - t0 > limit_ns) {
-      atomicExch(&g_moa_bf16_status, 6u);
-      return;
-    }
-  }
-}
-
-__device__ __forceinline__ float ex2_approx(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-// log2 by the MUFU lg2 instruction (absolute error about 2^-22 for the row sums l >= 1 used here).
-__device__ __forceinline__ float lg2_approx(float x) {
-  float y;
-  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);  // .x (low 16 bits) = lo
-  return *reinterpret_cast<uint32_t*>(&v);
-}
-
-// Packed fp32 pairs (Blackwell f32x2 ALU forms): one instruction for two lanes of data.
-__device__ __forceinline__ uint64_t pack_f32x2(float lo, float hi) {
-  uint64_t r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
-  return r;
-}
-// (d0, d1) = (a0, a1) * b + c, with b and c packed pairs.
-__device__ __forceinline__ void ffma2(float& d0, float& d1, float a0, float a1, uint64_t b,
-                                      uint64_t c) {
-  asm("{\n\t.reg .b64 ra, rd;\n\tmov.b64 ra, {%2, %3};\n\t"
-      "fma.rn.f32x2 rd, ra, %4, %5;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-      : "=f"(d0), "=f"(d1)
-      : "f"(a0), "f"(a1), "l"(b), "l"(c));
-}
-// (a0, a1) += (b0, b1).
-__device__ __forceinline__ void fadd2(float& a0, float& a1, float b0, float b1) {
-  asm("{\n\t.reg .b64 ra, rb, rd;\n\tmov.b64 ra, {%0, %1};\n\tmov.b64 rb, {%2, %3};\n\t"
-      "add.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-      : "+f"(a0), "+f"(a1)
-      : "f"(b0), "f"(b1));
-}
-__device__ __forceinline__ float max3f(float a, float b, float c) {
-  float d;
-  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
-  return d;
-}
 // Maximum of 128 values (of their negations if NEG) with four independent 3-input chains.
 template <bool NEG>
 __device__ __forceinline__ float row_max128(const float* s) {
@@ -216,19 +122,6 @@ __device__ __forceinline__ float row_max128(const float* s) {
   a0 = max3f(a0, v(124), v(125));
   a1 = max3f(a1, v(126), v(127));
   return max3f(a0, a1, fmaxf(a2, a3));
-}
-
-// Loads 128 fp32 columns of this thread's TMEM lane into s[] and waits for completion.
-__device__ __forceinline__ void tmem_load_row128(uint32_t taddr, uint32_t* s) {
-  tmem_ld_32x32b_x32(taddr + 0, s + 0);
-  tmem_ld_32x32b_x32(taddr + 32, s + 32);
-  tmem_ld_32x32b_x32(taddr + 64, s + 64);
-  tmem_ld_32x32b_x32(taddr + 96, s + 96);
-  tmem_wait_ld();
-  reg_anchor_x32(s + 0);
-  reg_anchor_x32(s + 32);
-  reg_anchor_x32(s + 64);
-  reg_anchor_x32(s + 96);
 }
 
 // Multiplies DV fp32 TMEM columns of this thread's lane by alpha (warp-collective).
@@ -286,7 +179,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   // This CTA's key blocks: [kb0, kb0 + n_kt) (all of them unless the key axis is split).
   const int kb0 = SPLIT ? split * kv_per_split : 0;
   const int n_kt = SPLIT ? min((Nk + kBN - 1) / kBN - kb0, kv_per_split) : (Nk + kBN - 1) / kBN;
-  const WaitCtl wc{abort_flag, wait_limit_ns, C::kSepP ? kWaitHintNs : 0u};
+  const WaitCtl wc{abort_flag, wait_limit_ns, C::kSepP ? kWaitHintNs : 0u, &g_moa_bf16_status};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
@@ -372,9 +265,10 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       }
       if (aborted || *abort_flag) {
         // Let every copy already issued land before the CTA can exit.
-        wait_quiesce(q_full, 0, wait_limit_ns);
+        wait_quiesce(q_full, 0, wait_limit_ns, &g_moa_bf16_status);
         for (int sl = 0; sl < C::kStages; ++sl)
-          if (issued & (1u << sl)) wait_quiesce(full_bar(sl), (issued_phase >> sl) & 1u, wait_limit_ns);
+          if (issued & (1u << sl))
+            wait_quiesce(full_bar(sl), (issued_phase >> sl) & 1u, wait_limit_ns, &g_moa_bf16_status);
       }
     }
   } else if (warp == kMmaWarp0 || warp == kMmaWarp1) {
@@ -704,8 +598,8 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
 
   // Teardown: wait for the tensor core to go quiet before freeing TMEM.
   if (warp == kMmaWarp0) {
-    wait_quiesce(o_done(0), 0, wait_limit_ns);
-    wait_quiesce(o_done(1), 0, wait_limit_ns);
+    wait_quiesce(o_done(0), 0, wait_limit_ns, &g_moa_bf16_status);
+    wait_quiesce(o_done(1), 0, wait_limit_ns, &g_moa_bf16_status);
   }
   tc_fence_before_sync();
   __syncthreads();
@@ -758,7 +652,7 @@ __global__ void __launch_bounds__(32, 1) wait_timeout_selftest_kernel(uint64_t l
   }
   __syncwarp();
   if (threadIdx.x == 0) {
-    const WaitCtl wc{&abort_flag, limit_ns, 0u};
+    const WaitCtl wc{&abort_flag, limit_ns, 0u, &g_moa_bf16_status};
     if (wait_bounded(smem_u32(&bar), 0, wc)) atomicExch(&g_moa_bf16_status, 0xBADu);
   }
 }
@@ -791,10 +685,14 @@ EncodeTiledFn get_encode_fn(char* msg, size_t msglen) {
   return fn;
 }
 
+}  // namespace
+
 // 3-D map over a contiguous [BH, N, d] bf16 tensor; box = 64 columns x 128 rows x 1 slice,
 // 128-byte swizzle.  Rows past N inside a slice read as zero (never the next slice).
-bool encode_map(EncodeTiledFn enc, CUtensorMap* map, const void* base, int64_t BH, int64_t N,
-                int64_t d, char* msg, size_t msglen) {
+bool encode_bf16_map(CUtensorMap* map, const void* base, int64_t BH, int64_t N, int64_t d,
+                     char* msg, size_t msglen) {
+  EncodeTiledFn enc = get_encode_fn(msg, msglen);
+  if (!enc) return false;
   const cuuint64_t dims[3] = {cuuint64_t(d), cuuint64_t(N), cuuint64_t(BH)};
   const cuuint64_t strides[2] = {cuuint64_t(d * 2), cuuint64_t(N * d * 2)};
   const cuuint32_t box[3] = {64, 128, 1};
@@ -809,6 +707,8 @@ bool encode_map(EncodeTiledFn enc, CUtensorMap* map, const void* base, int64_t B
   }
   return true;
 }
+
+namespace {
 
 template <int DK, int DV>
 int launch_tc(const AttnArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
@@ -890,13 +790,11 @@ int launch_attn_fwd_bf16(const AttnArgs& a, char* msg, size_t msglen) {
 
 int launch_attn_fwd_bf16_split(const AttnArgs& a, const SplitPlan& sp, void* ws, char* msg,
                                size_t msglen) {
-  EncodeTiledFn enc = get_encode_fn(msg, msglen);
-  if (!enc) return 5;
   const int64_t BH = a.B * a.H;
   CUtensorMap mq, mk, mv;
-  if (!encode_map(enc, &mq, a.Q, BH, a.Nq, a.dk, msg, msglen)) return 5;
-  if (!encode_map(enc, &mk, a.K, BH, a.Nk, a.dk, msg, msglen)) return 5;
-  if (!encode_map(enc, &mv, a.V, BH, a.Nk, a.dv, msg, msglen)) return 5;
+  if (!encode_bf16_map(&mq, a.Q, BH, a.Nq, a.dk, msg, msglen)) return 5;
+  if (!encode_bf16_map(&mk, a.K, BH, a.Nk, a.dk, msg, msglen)) return 5;
+  if (!encode_bf16_map(&mv, a.V, BH, a.Nk, a.dv, msg, msglen)) return 5;
   if (a.dk == 64 && a.dv == 64) return launch_tc<64, 64>(a, mq, mk, mv, sp, ws, msg, msglen);
   if (a.dk == 128 && a.dv == 128) return launch_tc<128, 128>(a, mq, mk, mv, sp, ws, msg, msglen);
   if (a.dk == 128 && a.dv == 64) return launch_tc<128, 64>(a, mq, mk, mv, sp, ws, msg, msglen);

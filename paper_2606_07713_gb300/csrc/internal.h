@@ -2,6 +2,7 @@
 #pragma once
 #include <cstddef>
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 namespace moa {
@@ -45,6 +46,35 @@ int launch_attn_fwd_bf16_split(const AttnArgs& a, const SplitPlan& sp, void* ws,
 // split whose partials exceed kNoallocScratchBytes with MOA_ERR_UNSUPPORTED_SHAPE).
 int launch_attn_fwd_bf16_split_noalloc(const AttnArgs& a, const SplitPlan& sp, char* msg,
                                        size_t msglen);
+
+// Tensor map over a contiguous bf16 [BH, N, d] tensor: box of 64 columns x 128 rows, 128-byte
+// swizzle, rows past N of a slice read as zero.  False (and a message) on failure.
+bool encode_bf16_map(CUtensorMap* map, const void* base, int64_t BH, int64_t N, int64_t d,
+                     char* msg, size_t msglen);
+
+// Validated arguments of one backward call (see include/moa_attn.h, moa_attn_bwd).
+struct BwdArgs {
+  const void* Q;
+  const void* K;
+  const void* V;
+  const void* O;
+  const void* dO;
+  const float* lse;
+  void* dQ;
+  void* dK;
+  void* dV;
+  int64_t B, H, Nq, Nk, dk, dv;
+  float scale;
+  void* ws;  // bwd_workspace_bytes(...) bytes, 16-byte aligned
+  cudaStream_t stream;
+};
+
+// Workspace of the bf16 backward: per (b,h) and padded query row, D = rowsum(dO * O) and the
+// log-sum-exp in log2 units, fp32.
+size_t bwd_workspace_bytes(int64_t B, int64_t H, int64_t Nq);
+int launch_attn_bwd_bf16(const BwdArgs& a, char* msg, size_t msglen);
+// Reads and clears the status word of the backward kernels' bounded waits (after a sync).
+cudaError_t bwd_read_and_clear_status(unsigned* value);
 
 // Launches the bounded-wait self test (a wait that nothing completes) on `stream`.
 cudaError_t launch_wait_timeout_selftest(uint64_t limit_ns, cudaStream_t stream);

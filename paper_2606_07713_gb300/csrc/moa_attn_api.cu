@@ -229,16 +229,72 @@ int moa_attn_fwd_splitkv_noalloc(const void* Q, const void* K, const void* V, vo
   return MOA_OK;
 }
 
+size_t moa_attn_bwd_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int64_t d_k,
+                                    int64_t d_v, int dtype) {
+  (void)N_k;
+  (void)d_k;
+  (void)d_v;
+  if (dtype != MOA_BF16 || B <= 0 || H <= 0 || N_q <= 0) return 0;
+  if (moa::numel4(B, H, N_q + 127, 8) < 0) return 0;
+  return moa::bwd_workspace_bytes(B, H, N_q);
+}
+
+int moa_attn_bwd(const void* Q, const void* K, const void* V, const void* O, const void* dO,
+                 const float* LSE, void* dQ, void* dK, void* dV, int64_t B, int64_t H,
+                 int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v, float scale, int dtype,
+                 void* workspace, size_t workspace_bytes, void* stream) {
+  if (!dO || !LSE || !dQ || !dK || !dV)
+    return moa::fail(MOA_ERR_INVALID_ARG, "null pointer among dO, LSE, dQ, dK, dV");
+  int64_t sz[4];
+  int rc = moa::validate(Q, K, V, const_cast<void*>(O), B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
+  if (rc != MOA_OK) return rc;
+  if (dtype != MOA_BF16)
+    return moa::fail(MOA_ERR_UNSUPPORTED_DTYPE, "the backward pass takes bf16 tensors only");
+  const void* al[5] = {dO, dQ, dK, dV, workspace};
+  for (const void* p : al)
+    if (reinterpret_cast<uintptr_t>(p) % 16 != 0)
+      return moa::fail(MOA_ERR_MISALIGNED, "pointer %p is not 16-byte aligned", p);
+  if (reinterpret_cast<uintptr_t>(LSE) % 4 != 0)
+    return moa::fail(MOA_ERR_MISALIGNED, "LSE pointer is not 4-byte aligned");
+  const size_t need = moa::bwd_workspace_bytes(B, H, N_q);
+  if (workspace == nullptr || workspace_bytes < need)
+    return moa::fail(MOA_ERR_INVALID_ARG, "workspace too small: need %zu bytes, got %zu", need,
+                     workspace == nullptr ? size_t(0) : workspace_bytes);
+  // Read-only: Q, K, V, O, dO, LSE.  Written: dQ, dK, dV, workspace (no two may overlap, and
+  // none may overlap a read-only buffer).
+  const void* ro[6] = {Q, K, V, O, dO, LSE};
+  const int64_t rosz[6] = {sz[0], sz[1], sz[2], sz[3], sz[3], B * H * N_q * 4};
+  const void* wr[4] = {dQ, dK, dV, workspace};
+  const int64_t wrsz[4] = {sz[0], sz[1], sz[2], int64_t(need)};
+  for (int i = 0; i < 4; ++i) {
+    for (int j = 0; j < 6; ++j)
+      if (moa::overlaps(wr[i], wrsz[i], ro[j], rosz[j]))
+        return moa::fail(MOA_ERR_INVALID_ARG, "an output or the workspace overlaps an input");
+    for (int j = i + 1; j < 4; ++j)
+      if (moa::overlaps(wr[i], wrsz[i], wr[j], wrsz[j]))
+        return moa::fail(MOA_ERR_INVALID_ARG, "outputs or the workspace overlap each other");
+  }
+  moa::BwdArgs a{Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v, scale, workspace,
+                 static_cast<cudaStream_t>(stream)};
+  char msg[256] = {0};
+  rc = moa::launch_attn_bwd_bf16(a, msg, sizeof(msg));
+  if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
+  moa::t_last_error[0] = '\0';
+  return MOA_OK;
+}
+
 const char* moa_last_error(void) { return moa::t_last_error; }
 
 int moa_get_device_status(void* stream) {
   cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess)
     return moa::fail(MOA_ERR_CUDA, "stream synchronize: %s", cudaGetErrorString(e));
-  unsigned v = 0;
+  unsigned v = 0, vb = 0;
   e = moa::bf16_read_and_clear_status(&v);
+  if (e == cudaSuccess) e = moa::bwd_read_and_clear_status(&vb);
   if (e != cudaSuccess)
     return moa::fail(MOA_ERR_CUDA, "status word read: %s", cudaGetErrorString(e));
+  v |= vb;
   if (v != 0)
     return moa::fail(MOA_ERR_DEVICE_TIMEOUT, "a kernel wait ran out (status %u)", v);
   return MOA_OK;

@@ -1,6 +1,6 @@
 // Inline-PTX building blocks for sm_103a: mbarriers, TMA tensor copies and the
 // fifth-generation tensor-core instructions (tcgen05: TMEM allocation, MMA,
-// commit, TMEM loads/stores).  Used only by the bf16 attention kernel.
+// commit, TMEM loads/stores).  Used by the bf16 tensor-core kernels.
 #pragma once
 #include <cstdint>
 #include <cuda.h>
@@ -97,6 +97,16 @@ __device__ __forceinline__ uint64_t l2_policy_evict_first() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
   return p;
+}
+
+// Non-tensor bulk copy global -> shared (both addresses 16-byte aligned, bytes a multiple of 16),
+// completion on an mbarrier.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes,
+                                          uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
+      : "memory");
 }
 
 // ---------------------------------------------------------------------------------------------

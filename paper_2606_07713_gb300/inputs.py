@@ -38,7 +38,7 @@ _M1 = np.uint64(0xBF58476D1CE4E5B9)
 _M2 = np.uint64(0x94D049BB133111EB)
 _CHUNK = 1 << 20
 
-STREAM_Q, STREAM_K, STREAM_V, STREAM_PLANT = 0, 1, 2, 3
+STREAM_Q, STREAM_K, STREAM_V, STREAM_PLANT, STREAM_DO = 0, 1, 2, 3, 4
 
 
 def _mix64(z: np.ndarray) -> np.ndarray:
@@ -275,6 +275,20 @@ def make_inputs(cfg: AttnConfig | int) -> AttnInputs:
                         qb[b, h, i, :] = kb[b, h, kk, :]
                     plants.append((b, h, i, kk))
     return AttnInputs(cfg, q, k, v, qb, kb, vb, tuple(plants))
+
+
+def make_grad_output(cfg: AttnConfig | int, sigma: float = 1.0):
+    """dL/dO for the backward pass: i.i.d. sigma * N(0,1) of O's shape [B, H, N_q, d_v], stored in
+    the workload's type.  Returns (values as float32, bf16 bit patterns or None)."""
+    if isinstance(cfg, int):
+        cfg = CONFIGS[cfg]
+    s = cfg.shape
+    g64 = normal(cfg.the_seed, STREAM_DO, s.numel_o)
+    if sigma != 1.0:
+        g64 *= sigma
+    g, gb = _store(g64, cfg.dtype)
+    shape = (s.B, s.H, s.N_q, s.d_v)
+    return g.reshape(shape), (gb.reshape(shape) if gb is not None else None)
 
 
 def custom_config(B, H, N_q, N_k, d_k, d_v, dtype="bf16", seed=1234, q_sigma=1.0,

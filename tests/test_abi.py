@@ -122,3 +122,42 @@ def test_lse_validation_without_gpu(L):
     assert f(A, B_, C, D, A, *ok_args) == _lib.MOA_ERR_INVALID_ARG           # LSE aliases Q
     assert f(None, B_, C, D, E, *ok_args) == _lib.MOA_ERR_INVALID_ARG        # the usual checks too
     assert f(A, B_, C, D, E, 1, 1, 8, 8, 96, 64, 0.125, 1, None) == _lib.MOA_ERR_UNSUPPORTED_SHAPE
+
+
+def test_bwd_workspace_formula(L):
+    ws = pkg.moa_attn_bwd_workspace_bytes
+    assert ws(2, 3, 200, 300, 64, 64, pkg.MOA_BF16) == 2 * 2 * 3 * 256 * 4
+    assert ws(1, 1, 128, 5, 128, 64, pkg.MOA_BF16) == 2 * 128 * 4
+    assert ws(1, 1, 128, 5, 128, 64, pkg.MOA_FP32) == 0
+    assert ws(0, 1, 128, 5, 128, 64, pkg.MOA_BF16) == 0
+
+
+def test_bwd_validation_without_gpu(L):
+    f = _lib.moa_attn_bwd
+    # Q, K, V, O, dO, LSE, dQ, dK, dV, workspace: fake addresses 1 MiB apart
+    P = [0x1000000 * (i + 1) for i in range(10)]
+    dims = (1, 1, 8, 8, 64, 64, 0.125)
+
+    def call(ptrs=None, dtype=1, ws_bytes=1 << 20, d=dims):
+        p = list(P if ptrs is None else ptrs)
+        return f(*p[:9], *d, dtype, p[9], ws_bytes, None)
+
+    for i in range(4, 9):  # null dO, LSE or an output
+        q = list(P)
+        q[i] = None
+        assert call(q) == _lib.MOA_ERR_INVALID_ARG
+    assert call(dtype=0) == _lib.MOA_ERR_UNSUPPORTED_DTYPE
+    assert call(d=(1, 1, 8, 8, 96, 64, 0.125)) == _lib.MOA_ERR_UNSUPPORTED_SHAPE
+    assert call(ws_bytes=100) == _lib.MOA_ERR_INVALID_ARG               # workspace too small
+    q = list(P); q[9] = None
+    assert call(q) == _lib.MOA_ERR_INVALID_ARG                          # no workspace
+    q = list(P); q[6] = P[6] + 8
+    assert call(q) == _lib.MOA_ERR_MISALIGNED                           # dQ misaligned
+    q = list(P); q[5] = P[5] + 2
+    assert call(q) == _lib.MOA_ERR_MISALIGNED                           # LSE misaligned
+    q = list(P); q[7] = P[0]
+    assert call(q) == _lib.MOA_ERR_INVALID_ARG                          # dK aliases Q
+    q = list(P); q[8] = P[6]
+    assert call(q) == _lib.MOA_ERR_INVALID_ARG                          # dV aliases dQ
+    q = list(P); q[9] = P[4]
+    assert call(q) == _lib.MOA_ERR_INVALID_ARG                          # workspace aliases dO

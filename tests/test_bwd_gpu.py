@@ -1,0 +1,117 @@
+"""Backward pass (moa_attn_bwd) vs the fp64 oracle, element by element, through the C ABI.
+
+The GPU path takes O and LSE from its own forward kernel (moa_attn_fwd_lse); the oracle
+recomputes everything in fp64 from Q, K, V and dO.  Tolerance: the bf16 bound of the forward
+tests, max|g - g_ref| <= 2e-2 * max|g_ref| per gradient.  A model of the bf16 roundings the
+kernels make (O, the weights W and dS rounded to bf16 before the products) gives 1.4e-3 to
+2.9e-3 on these shapes, so the bound has a margin of about 7.
+"""
+import numpy as np
+import pytest
+
+from gpu_helpers import BF16_TOL, rel_err, to_device
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+import paper_2606_07713_gb300 as pkg  # noqa: E402
+from paper_2606_07713_gb300 import inputs as I  # noqa: E402
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _need_gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    pkg.lib()
+
+
+def bf16_dev(bits):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to("cuda:0")
+
+
+def run_bwd(x, g_bits, scale=None):
+    scale = x.scale if scale is None else scale
+    q, k, v = to_device(x)
+    do = bf16_dev(g_bits)
+    o, lse = pkg.attn_fwd_lse(q, k, v, scale)
+    dq, dk, dv = pkg.attn_bwd(q, k, v, o, lse, do, scale)
+    torch.cuda.synchronize()
+    pkg.check(pkg.get_device_status())
+    return tuple(t.float().cpu().numpy() for t in (dq, dk, dv))
+
+
+def check_grads(got, ref, what):
+    for name, a, b in zip(("dQ", "dK", "dV"), got, ref):
+        assert np.all(np.isfinite(a)), f"{what} {name}: non-finite"
+        if np.max(np.abs(b)) == 0.0:
+            # an exactly zero gradient (one key): only the rounding of dP - D remains
+            assert np.max(np.abs(a)) <= 1e-3, f"{what} {name}: {np.max(np.abs(a)):.3e} for 0"
+            continue
+        err = rel_err(a, b)
+        assert err <= BF16_TOL, f"{what} {name}: max|g-g_ref|/max|g_ref| = {err:.3e}"
+
+
+SHAPES = [
+    (1, 1, 128, 128, 64, 64),
+    (1, 1, 256, 256, 128, 128),
+    (2, 3, 200, 300, 128, 128),
+    (1, 2, 300, 1000, 64, 64),
+    (1, 2, 300, 1000, 64, 128),
+    (2, 2, 513, 777, 128, 64),
+    (1, 1, 1000, 129, 64, 64),
+    (3, 1, 130, 2048, 128, 128),
+    (1, 1, 5, 3, 64, 64),
+    (1, 1, 1, 1, 128, 128),
+]
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: "x".join(map(str, s)))
+def test_bwd_parity(oracle, shape):
+    cfg = I.custom_config(*shape, dtype="bf16", seed=sum(shape) + 11)
+    x = I.make_inputs(cfg)
+    g, gb = I.make_grad_output(cfg)
+    got = run_bwd(x, gb)
+    ref = oracle.attn_bwd(x.q, x.k, x.v, g, x.scale)
+    check_grads(got, ref, str(shape))
+
+
+@pytest.mark.parametrize("scale", [-0.3, 2.0 / 8])
+def test_bwd_other_scales(oracle, scale):
+    cfg = I.custom_config(1, 2, 150, 260, 64, 64, dtype="bf16", seed=93)
+    x = I.make_inputs(cfg)
+    g, gb = I.make_grad_output(cfg)
+    got = run_bwd(x, gb, scale)
+    check_grads(got, oracle.attn_bwd(x.q, x.k, x.v, g, scale), f"scale {scale}")
+
+
+def test_bwd_large_scores_and_planted_rows(oracle):
+    cfg = I.custom_config(1, 2, 384, 700, 128, 128, dtype="bf16", seed=19, q_sigma=4.0,
+                          plants_per_head=4)
+    x = I.make_inputs(cfg)
+    g, gb = I.make_grad_output(cfg)
+    check_grads(run_bwd(x, gb), oracle.attn_bwd(x.q, x.k, x.v, g, x.scale), "large scores")
+
+
+def test_bwd_single_key_closed_form():
+    """One key: the weights are all 1, so dQ = dK = 0 up to the rounding of dP - D, and
+    dV = sum over the query rows of dO."""
+    cfg = I.custom_config(1, 2, 300, 1, 64, 64, dtype="bf16", seed=7)
+    x = I.make_inputs(cfg)
+    g, gb = I.make_grad_output(cfg)
+    dq, dk, dv = run_bwd(x, gb)
+    assert np.max(np.abs(dq)) <= 1e-2 and np.max(np.abs(dk)) <= 1e-1
+    ref = g.astype(np.float64).sum(axis=2)
+    assert rel_err(dv[:, :, 0], ref) <= 1e-2
+
+
+def test_bwd_gradients_sum_rules():
+    """Properties at a size the oracle would be slow on: each head's dK rows sum to ~0 and its
+    dV rows to sum_i dO_i (weights sum to one per row)."""
+    cfg = I.custom_config(1, 4, 2048, 2048, 64, 64, dtype="bf16", seed=29)
+    x = I.make_inputs(cfg)
+    g, gb = I.make_grad_output(cfg)
+    dq, dk, dv = run_bwd(x, gb)
+    gsum = g.astype(np.float64).sum(axis=2)
+    assert rel_err(dv.astype(np.float64).sum(axis=2), gsum) <= 2e-2
+    assert np.max(np.abs(dk.astype(np.float64).sum(axis=2))) <= 2e-2 * np.max(np.abs(dk)) * np.sqrt(2048)
