@@ -5,7 +5,7 @@ N(0,1) from the seeded generator, scale=1/sqrt(d_k), no mask.  One step = one at
 forward over that batch (the whole hot path: one kernel launch).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference|classical]
-                    [--workload ID] [--shape B,H,N_q,N_k,d_k,d_v]
+                    [--workload ID] [--shape B,H,N_q,N_k,d_k,d_v] [--pass fwd|bwd]
 
 Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s: FLOPs of every step on every
 rank divided by the slowest rank's summed kernel time, measured with CUDA events on the
@@ -16,7 +16,8 @@ rows per step).  `--impl classical` times the step-by-step path whose traffic th
 M_classical models (Section 8.2): the score matrix, its max-shifted exponentials and the
 normalised weights each materialised in device memory by eager PyTorch ops (cuBLAS GEMMs and
 elementwise/reduction kernels) -- a measurement of the comparison, not part of the library.
-`--shape` replaces the workload's sizes (bf16, same generator) for traffic sweeps.  Multi-GPU (torchrun): every rank runs its own full copy of the workload (the
+`--shape` replaces the workload's sizes (bf16, same generator) for traffic sweeps.  `--pass bwd`
+times moa_attn_bwd (three launches) on the same workload instead of the forward pass.  Multi-GPU (torchrun): every rank runs its own full copy of the workload (the
 (b, h) problems are independent; no collective on the data path), so scaling is weak.
 """
 from __future__ import annotations
@@ -304,6 +305,159 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
 
 
 # ------------------------------------------------------------------------------------------
+# the backward pass (--pass bwd)
+# ------------------------------------------------------------------------------------------
+def bwd_flops(s: I.AttnShape) -> float:
+    """Algorithmic FLOPs of one backward pass: the five products S = Q K^T (rebuilt), dP = dO V^T,
+    dV = W^T dO, dQ = dS K, dK = dS^T Q."""
+    return 2.0 * s.B * s.H * s.N_q * s.N_k * (3 * s.d_k + 2 * s.d_v)
+
+
+def bwd_bytes(s: I.AttnShape) -> float:
+    """Compulsory HBM bytes of one bf16 backward pass: read Q, K, V, O, dO, LSE once, write
+    dQ, dK, dV once."""
+    bh = s.B * s.H
+    reads = 2.0 * (s.N_q * s.d_k + s.N_k * s.d_k + s.N_k * s.d_v + 2 * s.N_q * s.d_v) + 4.0 * s.N_q
+    writes = 2.0 * (s.N_q * s.d_k + s.N_k * s.d_k + s.N_k * s.d_v)
+    return bh * (reads + writes)
+
+
+def cpu_baseline_bwd(cfg, x, g, budget_s: float = 12.0) -> dict:
+    import oracle
+    orc = oracle.get()
+    s = cfg.shape
+    bh = s.B * s.H
+    per_slice = bwd_flops(I.AttnShape(1, 1, s.N_q, s.N_k, s.d_k, s.d_v))
+    q = x.q.reshape(bh, 1, s.N_q, s.d_k)
+    k = x.k.reshape(bh, 1, s.N_k, s.d_k)
+    v = x.v.reshape(bh, 1, s.N_k, s.d_v)
+    gg = g.reshape(bh, 1, s.N_q, s.d_v)
+    n = min(bh, orc.max_threads())
+    t0 = time.perf_counter()
+    orc.attn_bwd(q[:n], k[:n], v[:n], gg[:n], cfg.scale)
+    dt = time.perf_counter() - t0
+    if dt < budget_s / 4 and n < bh:
+        n2 = int(min(bh, max(n, n * budget_s / max(dt, 1e-6) / 2)))
+        t0 = time.perf_counter()
+        orc.attn_bwd(q[:n2], k[:n2], v[:n2], gg[:n2], cfg.scale)
+        dt, n = time.perf_counter() - t0, n2
+    return {"value": round(per_slice * n / dt / 1e12, 6), "unit": "TFLOP/s",
+            "cores": orc.max_threads(), "kind": "oracle",
+            "sample": f"{n} of {bh} (b,h) slices, whole backward in fp64, {dt:.1f} s"}
+
+
+def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
+    import torch
+    import torch.distributed as dist
+
+    import paper_2606_07713_gb300 as pkg
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    pkg.lib()
+    s = cfg.shape
+    if cfg.dtype != "bf16":
+        raise SystemExit("the backward pass takes bf16 workloads")
+    x = I.make_inputs(cfg)
+    g, gbits = I.make_grad_output(cfg)
+    q, k, v, do = (to_device_bf16(b, dev) for b in (x.q_bits, x.k_bits, x.v_bits, gbits))
+    o, lse = pkg.attn_fwd_lse(q, k, v, cfg.scale)
+    ws = torch.empty(pkg.moa_attn_bwd_workspace_bytes(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v,
+                                                      pkg.MOA_BF16), dtype=torch.uint8, device=dev)
+    host = [t.cpu().pin_memory() for t in (q, k, v, o, do, lse)]
+    host_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in (q, k, v)]
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flops = bwd_flops(s)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        pkg.attn_bwd(q, k, v, o, lse, do, cfg.scale, workspace=ws)
+    torch.cuda.synchronize(dev)
+    pkg.check(pkg.get_device_status())
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    barrier()
+    for i in range(args.steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        pkg.attn_bwd(q, k, v, o, lse, do, cfg.scale, workspace=ws, stream=stream)
+        ev[i][1].record(stream)
+    barrier()
+    kern_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = float(np.sum(kern_ms))
+    # end to end: the forward's outputs and dO from pinned host memory, gradients back
+    dq_, dk_, dv_ = (torch.empty_like(t) for t in (q, k, v))
+    dev_in = [torch.empty_like(t) for t in (q, k, v, o, do, lse)]
+    ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    barrier()
+    for i in range(args.steps):
+        flush.zero_()
+        ev2[i][0].record(stream)
+        for d_, h_ in zip(dev_in, host):
+            d_.copy_(h_, non_blocking=True)
+        grads = pkg.attn_bwd(*dev_in[:4], dev_in[5], dev_in[4], cfg.scale, workspace=ws, stream=stream)
+        for h_, d_ in zip(host_out, grads):
+            h_.copy_(d_, non_blocking=True)
+        ev2[i][1].record(stream)
+    barrier()
+    clocks = sampler.stop()
+    e2e_ms = float(np.sum([a.elapsed_time(b) for a, b in ev2]))
+    pkg.check(pkg.get_device_status())
+    total_ms, e2e_ms = reduce_max_over_ranks([total_ms, e2e_ms], device=dev)
+    if rank == 0:
+        peaks, peak_src = measured_peaks()
+        value = whole_job_tflops(flops, args.steps, world, total_ms)
+        achieved = flops / (float(np.mean(kern_ms)) * 1e-3) / 1e12
+        peak = float(peaks["bf16_tflops"])
+        line = {
+            "metric": "attention bwd TFLOP/s (algorithmic: 5 products) and % of GB300 bf16 peak",
+            "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 6),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic: seeded splitmix64 + Box-Muller inputs and dO of the workload's shape",
+            "config": dict(workload_desc(cfg), **{
+                "workload": workload_desc(cfg)["workload"].replace("SDPA fwd", "SDPA bwd"),
+                "pass": "backward (moa_attn_bwd)"}),
+            "compulsory_bytes": bwd_bytes(s),
+            "roofline": {
+                "bound": "tensor", "achieved": round(achieved, 2), "peak": peak,
+                "peak_source": f"{peak_src} bf16_tflops (burst; call timed alone)",
+                "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": None,
+                "kernel": "moa_attn_bwd: attn_bwd_pre + attn_bwd_dkdv + attn_bwd_dq (one call)",
+            },
+            "e2e": {
+                "value": round(whole_job_tflops(flops, args.steps, world, e2e_ms), 2),
+                "unit": "TFLOP/s",
+                "h2d_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host)),
+                "d2h_bytes_per_step": int(sum(t.numel() * t.element_size() for t in host_out)),
+                "api": "attn_bwd with host copies of Q, K, V, O, dO, LSE and the gradients",
+            },
+            "gpu_launches": 3 * args.steps,
+            "clocks": clocks,
+        }
+        if world == 1:
+            line["cpu_baseline"] = cpu_baseline_bwd(cfg, x, g, budget_s=args.cpu_budget)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+# ------------------------------------------------------------------------------------------
 # the classical path (what Eq. M_classical counts), for the measured traffic comparison
 # ------------------------------------------------------------------------------------------
 def classical_step(q, k, v, scale):
@@ -461,6 +615,8 @@ def main():
     ap.add_argument("--workload", type=int, default=DEFAULT_WORKLOAD, choices=sorted(I.CONFIGS))
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle time for the cpu_baseline sample")
+    ap.add_argument("--pass", dest="which", choices=["fwd", "bwd"], default="fwd",
+                    help="time the forward (default) or the backward pass")
     ap.add_argument("--shape", default=None,
                     help="B,H,N_q,N_k,d_k,d_v: a bf16 workload of this shape instead of --workload")
     args = ap.parse_args()
@@ -476,6 +632,8 @@ def main():
         run_reference(args, cfg)
     elif args.impl == "classical":
         run_classical(args, cfg)
+    elif args.which == "bwd":
+        run_ours_bwd(args, cfg)
     else:
         run_ours(args, cfg)
 
