@@ -71,7 +71,9 @@ def _load(path: str | None = None):
         lib.moa_oracle_attn_bwd_f64.argtypes = [f32p, f32p, f32p, f32p, f64p, f64p, f64p, i64,
                                                 i64, i64, i64, i64, i64, ctypes.c_double,
                                                 ctypes.c_int]
-        for name in ("moa_oracle_attn_bwd_f64", "moa_oracle_attn_lse_f64", "moa_oracle_attn_f64", "moa_oracle_rows_f64", "moa_oracle_weights_f64",
+        lib.moa_oracle_qkv_proj_f64.argtypes = [f32p, f32p, f64p, f64p, f64p, i64, i64, i64, i64,
+                                                i64, i64, ctypes.c_int]
+        for name in ("moa_oracle_qkv_proj_f64", "moa_oracle_attn_bwd_f64", "moa_oracle_attn_lse_f64", "moa_oracle_attn_f64", "moa_oracle_rows_f64", "moa_oracle_weights_f64",
                      "moa_oracle_scores_f64", "moa_oracle_attn_shifted_f64",
                      "moa_oracle_max_threads"):
             getattr(lib, name).restype = ctypes.c_int
@@ -225,6 +227,24 @@ class Oracle:
         if squeeze:
             return dq[0, 0], dkk[0, 0], dvv[0, 0]
         return dq, dkk, dvv
+
+    def qkv_proj(self, x, w, H: int, dk: int, dv: int, nthreads: int = 0):
+        """(Q, K, V) = X W_Q, X W_K, X W_V in fp64, head-major [B, H, N, d]; x [B, N, d_model],
+        w [d_model, 2*H*dk + H*dv] (W_Q | W_K | W_V)."""
+        B, N, d = np.shape(x)
+        if tuple(np.shape(w)) != (d, 2 * H * dk + H * dv):
+            raise ValueError(f"w must be {(d, 2 * H * dk + H * dv)}, got {np.shape(w)}")
+        x, xp = self._f32(x)
+        w, wp = self._f32(w)
+        q = np.empty((B, H, N, dk), dtype=np.float64)
+        k = np.empty((B, H, N, dk), dtype=np.float64)
+        v = np.empty((B, H, N, dv), dtype=np.float64)
+        dp = ctypes.POINTER(ctypes.c_double)
+        rc = self.lib.moa_oracle_qkv_proj_f64(xp, wp, q.ctypes.data_as(dp), k.ctypes.data_as(dp),
+                                              v.ctypes.data_as(dp), B, N, d, H, dk, dv,
+                                              int(nthreads))
+        self._check(rc, "moa_oracle_qkv_proj_f64")
+        return q, k, v
 
     def max_threads(self) -> int:
         return int(self.lib.moa_oracle_max_threads())

@@ -27,8 +27,9 @@
  * same on x86-64 and AArch64.  OpenMP splits the work over whole rows only, so
  * the result is bit-identical for any thread count.
  *
- * moa_oracle_attn_lse_f64 also returns each row's log-sum-exp, and moa_oracle_attn_bwd_f64
- * the gradients dQ, dK, dV of the backward pass (Stage 5, Section 9) for a given dL/dO.
+ * moa_oracle_attn_lse_f64 also returns each row's log-sum-exp, moa_oracle_attn_bwd_f64 the
+ * gradients dQ, dK, dV of the backward pass (Stage 5, Section 9) for a given dL/dO, and
+ * moa_oracle_qkv_proj_f64 the input projections Q = X W_Q, K = X W_K, V = X W_V (Section 4.1).
  *
  * Inputs are float32 arrays holding the stored values exactly (bf16 and fp32
  * values both embed exactly in float32); every element is widened to double
@@ -316,6 +317,49 @@ int moa_oracle_attn_bwd_f64(const float *Q, const float *K, const float *V, cons
         }
     }
     return status;
+}
+
+/*
+ * Input projections of Section 4.1: Q = X W_Q, K = X W_K, V = X W_V, for X [B, N, d] and the
+ * three weight matrices side by side in one row-major array W [d, H*dk + H*dk + H*dv]
+ * (columns [0, H*dk) are W_Q, then W_K, then W_V).  Column h*dk + j of W_Q produces feature j
+ * of head h, and the results are stored head-major, as the attention entry points take them:
+ *     Q[b,h,n,j] = sum_c X[b,n,c] W[c, h*dk + j]
+ *     K[b,h,n,j] = sum_c X[b,n,c] W[c, H*dk + h*dk + j]
+ *     V[b,h,n,j] = sum_c X[b,n,c] W[c, 2*H*dk + h*dv + j]
+ * Plain fp64 dot products in index order.
+ */
+int moa_oracle_qkv_proj_f64(const float *X, const float *W, double *Q, double *K, double *V,
+                            int64_t B, int64_t N, int64_t d, int64_t H, int64_t dk, int64_t dv,
+                            int nthreads)
+{
+    if (!X || !W || !Q || !K || !V) return -1;
+    if (B <= 0 || N <= 0 || d <= 0 || H <= 0 || dk <= 0 || dv <= 0) return -1;
+    const int64_t ncol = 2 * H * dk + H * dv;
+#ifdef _OPENMP
+    if (nthreads <= 0) nthreads = omp_get_max_threads();
+#pragma omp parallel for schedule(dynamic, 16) num_threads(nthreads)
+#endif
+    for (int64_t t = 0; t < B * N; ++t) {
+        const int64_t b = t / N, n = t % N;
+        const float *x = X + t * d;
+        for (int64_t col = 0; col < ncol; ++col) {
+            double acc = 0.0;
+            for (int64_t c = 0; c < d; ++c)
+                acc += (double)x[c] * (double)W[c * ncol + col];
+            if (col < H * dk) {
+                const int64_t h = col / dk, j = col % dk;
+                Q[((b * H + h) * N + n) * dk + j] = acc;
+            } else if (col < 2 * H * dk) {
+                const int64_t h = (col - H * dk) / dk, j = (col - H * dk) % dk;
+                K[((b * H + h) * N + n) * dk + j] = acc;
+            } else {
+                const int64_t h = (col - 2 * H * dk) / dv, j = (col - 2 * H * dk) % dv;
+                V[((b * H + h) * N + n) * dv + j] = acc;
+            }
+        }
+    }
+    return 0;
 }
 
 /* Threads an OpenMP region would use by default (1 without OpenMP). */

@@ -406,6 +406,48 @@ def pin_bwd_invariants(o):
                                                     o.attn_bwd(Q, K, V, G1, 0.3, nthreads=3)))
 
 
+# ----------------------------------------------------------------------------------------------
+# 5. Input projections (Section 4.1): Q = X W_Q, K = X W_K, V = X W_V, stored head-major
+# ----------------------------------------------------------------------------------------------
+def pin_qkv_proj_exact_integers(o):
+    """Small-integer X and W: every product and sum is exact, so the oracle must equal an
+    integer brute force (Python ints) in the documented head-major layout."""
+    r = _rng(500)
+    B, N, d, H, dk, dv = 2, 5, 6, 3, 2, 4
+    X = r.integers(-4, 5, size=(B, N, d))
+    W = r.integers(-4, 5, size=(d, 2 * H * dk + H * dv))
+    q, k, v = o.qkv_proj(_f32(X), _f32(W), H, dk, dv)
+    for b in range(B):
+        for n in range(N):
+            for h in range(H):
+                for j in range(dk):
+                    eq = sum(int(X[b, n, c]) * int(W[c, h * dk + j]) for c in range(d))
+                    ek = sum(int(X[b, n, c]) * int(W[c, H * dk + h * dk + j]) for c in range(d))
+                    assert q[b, h, n, j] == eq and k[b, h, n, j] == ek
+                for j in range(dv):
+                    ev = sum(int(X[b, n, c]) * int(W[c, 2 * H * dk + h * dv + j]) for c in range(d))
+                    assert v[b, h, n, j] == ev
+
+
+def pin_qkv_proj_unit_columns(o):
+    """W with one 1 per output column selects an input feature: the output must be that
+    feature of X, at the head and position the column names (catches layout mix-ups)."""
+    r = _rng(501)
+    B, N, d, H, dk, dv = 2, 7, 9, 2, 3, 2
+    X = _f32(r.normal(size=(B, N, d)))
+    ncol = 2 * H * dk + H * dv
+    src = r.integers(0, d, size=ncol)
+    W = np.zeros((d, ncol), dtype=np.float32)
+    W[src, np.arange(ncol)] = 1.0
+    q, k, v = o.qkv_proj(X, W, H, dk, dv)
+    for h in range(H):
+        for j in range(dk):
+            assert np.array_equal(q[:, h, :, j], X[:, :, src[h * dk + j]])
+            assert np.array_equal(k[:, h, :, j], X[:, :, src[H * dk + h * dk + j]])
+        for j in range(dv):
+            assert np.array_equal(v[:, h, :, j], X[:, :, src[2 * H * dk + h * dv + j]])
+
+
 ALL_PINS = [
     pin_paper_example,
     pin_decimal_bruteforce,
@@ -425,4 +467,6 @@ ALL_PINS = [
     pin_bwd_finite_differences,
     pin_bwd_closed_forms,
     pin_bwd_invariants,
+    pin_qkv_proj_exact_integers,
+    pin_qkv_proj_unit_columns,
 ]

@@ -41,6 +41,12 @@ MUTANTS = {
                        "dVh[k * dv + c] += dS[k] * (double)g[c];"),
     "bwd_dp_v_transposed": ("acc += (double)g[c] * (double)Vh[k * dv + c];",
                             "acc += (double)g[c] * (double)Vh[c * Nk + k];"),
+    "proj_columns_shifted": ("acc += (double)x[c] * (double)W[c * ncol + col];",
+                             "acc += (double)x[c] * (double)W[c * ncol + (col + H * dk) % ncol];"),
+    "proj_head_feature_swapped": ("const int64_t h = col / dk, j = col % dk;",
+                                  "const int64_t j = col / dk % dk, h = col % dk % H;"),
+    "proj_w_transposed": ("acc += (double)x[c] * (double)W[c * ncol + col];",
+                          "acc += (double)x[c] * (double)W[(col % d) * ncol + c];"),
     "bwd_dq_uses_q": ("acc += dS[k] * (double)Kh[k * dk + j];",
                       "acc += dS[k] * (double)Kh[j];"),
 }
