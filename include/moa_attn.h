@@ -146,6 +146,31 @@ size_t moa_attn_bwd_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N
                                     int64_t d_v, int dtype);
 
 /*
+ * moa_qkv_proj -- the input projections Q = X W_Q, K = X W_K, V = X W_V in one pass.
+ *
+ * Defines: paper Section 4.1 (the problem setup: Q, K, V are the input sequence X projected
+ * by learned weight matrices).  With the three weight matrices side by side in W,
+ *     Q[b,h,n,j] = sum_c X[b,n,c] W[c, h*d_k + j]
+ *     K[b,h,n,j] = sum_c X[b,n,c] W[c, H*d_k + h*d_k + j]
+ *     V[b,h,n,j] = sum_c X[b,n,c] W[c, 2*H*d_k + h*d_v + j]
+ * One tensor-core GEMM over all B*N tokens (X read once for all three); its epilogue stores
+ * each result in the head-major layout moa_attn_fwd takes, so no permute copy follows.
+ *
+ * Arguments:
+ *   X  device, [B, N, d_model] row-major, bf16, read only
+ *   W  device, [d_model, 2*H*d_k + H*d_v] row-major, bf16 (columns W_Q | W_K | W_V), read only
+ *   Q, K  device, written: [B, H, N, d_k];  V  device, written: [B, H, N, d_v]
+ *   dtype  MOA_BF16 only; fp32 accumulation, outputs rounded to bf16 once
+ *   stream a cudaStream_t of the current device
+ * Supported sizes: d_k, d_v in {64, 128}; d_model a multiple of 8; B*N < 2^31.  Alignment:
+ * all pointers 16-byte aligned.  Q, K, V must not overlap each other, X or W.
+ * Behaviour: asynchronous, one launch, allocates nothing; bounded waits as moa_attn_fwd.
+ * (The paper has no bias term and none is added.)
+ */
+int moa_qkv_proj(const void* X, const void* W, void* Q, void* K, void* V, int64_t B, int64_t N,
+                 int64_t d_model, int64_t H, int64_t d_k, int64_t d_v, int dtype, void* stream);
+
+/*
  * moa_attn_fwd_staged -- the same computation with host-resident inputs and output.
  *
  * Defines: as moa_attn_fwd (paper Section 4.1, Eq. attention).  Copies hQ, hK,

@@ -17,14 +17,15 @@ from ._lib import (MOA_BF16, MOA_FP32, MoaError, check, lib, moa_attn_dnf_bytes,
                    moa_attn_flops, moa_attn_fwd, moa_attn_fwd_staged, moa_attn_version,
                    moa_get_device_status, moa_last_error, moa_selftest_wait_timeout,
                    moa_attn_fwd_splitkv, moa_attn_splitkv_workspace_bytes, moa_attn_fwd_lse,
-                   moa_attn_bwd, moa_attn_bwd_workspace_bytes)
+                   moa_attn_bwd, moa_attn_bwd_workspace_bytes, moa_qkv_proj)
 
 __all__ = ["attn_fwd", "attn_fwd_staged", "get_device_status", "attn_flops", "dnf_bytes",
            "MOA_FP32", "MOA_BF16", "MoaError", "moa_attn_fwd", "moa_attn_fwd_staged",
            "moa_last_error", "moa_get_device_status", "moa_attn_flops", "moa_attn_dnf_bytes",
            "moa_attn_version", "moa_selftest_wait_timeout", "attn_fwd_splitkv",
            "moa_attn_fwd_splitkv", "moa_attn_splitkv_workspace_bytes", "attn_fwd_lse",
-           "moa_attn_fwd_lse", "attn_bwd", "moa_attn_bwd", "moa_attn_bwd_workspace_bytes"]
+           "moa_attn_fwd_lse", "attn_bwd", "moa_attn_bwd", "moa_attn_bwd_workspace_bytes",
+           "qkv_proj", "moa_qkv_proj"]
 
 
 def _dtype_code(t) -> int:
@@ -135,6 +136,33 @@ def attn_bwd(q, k, v, o, lse, do, scale: float | None = None, workspace=None, st
                            Nk, dk, dv, float(scale), code, workspace.data_ptr(), workspace.numel(),
                            s.cuda_stream))
     return dq, dkk, dvv
+
+
+def qkv_proj(x, w, H: int, d_k: int, d_v: int, out=None, stream=None):
+    """(Q, K, V) = (X W_Q, X W_K, X W_V) in head-major layout [B, H, N, d] from x [B, N, d_model]
+    and w [d_model, 2*H*d_k + H*d_v] (W_Q | W_K | W_V), bf16 CUDA tensors."""
+    import torch
+    for t in (x, w):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError("qkv_proj needs contiguous CUDA tensors")
+    if x.dim() != 3 or w.dim() != 2:
+        raise ValueError("x must be [B, N, d_model] and w [d_model, 2*H*d_k + H*d_v]")
+    if x.dtype != w.dtype:
+        raise TypeError("x and w must share one dtype")
+    code = _dtype_code(x)
+    B, N, d = x.shape
+    if tuple(w.shape) != (d, 2 * H * d_k + H * d_v):
+        raise ValueError(f"w must be {(d, 2 * H * d_k + H * d_v)}, got {tuple(w.shape)}")
+    if out is None:
+        out = (torch.empty((B, H, N, d_k), dtype=x.dtype, device=x.device),
+               torch.empty((B, H, N, d_k), dtype=x.dtype, device=x.device),
+               torch.empty((B, H, N, d_v), dtype=x.dtype, device=x.device))
+    q, k, v = out
+    with torch.cuda.device(x.device):
+        s = stream if stream is not None else torch.cuda.current_stream(x.device)
+        check(moa_qkv_proj(x.data_ptr(), w.data_ptr(), q.data_ptr(), k.data_ptr(), v.data_ptr(),
+                           B, N, d, H, d_k, d_v, code, s.cuda_stream))
+    return q, k, v
 
 
 def attn_fwd_splitkv(q, k, v, num_splits: int, scale: float | None = None, out=None,

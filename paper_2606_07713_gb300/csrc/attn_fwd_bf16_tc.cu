@@ -691,11 +691,16 @@ EncodeTiledFn get_encode_fn(char* msg, size_t msglen) {
 // 128-byte swizzle.  Rows past N inside a slice read as zero (never the next slice).
 bool encode_bf16_map(CUtensorMap* map, const void* base, int64_t BH, int64_t N, int64_t d,
                      char* msg, size_t msglen) {
+  return encode_bf16_map_box(map, base, BH, N, d, 128, msg, msglen);
+}
+
+bool encode_bf16_map_box(CUtensorMap* map, const void* base, int64_t BH, int64_t N, int64_t d,
+                         int box_rows, char* msg, size_t msglen) {
   EncodeTiledFn enc = get_encode_fn(msg, msglen);
   if (!enc) return false;
   const cuuint64_t dims[3] = {cuuint64_t(d), cuuint64_t(N), cuuint64_t(BH)};
   const cuuint64_t strides[2] = {cuuint64_t(d * 2), cuuint64_t(N * d * 2)};
-  const cuuint32_t box[3] = {64, 128, 1};
+  const cuuint32_t box[3] = {64, cuuint32_t(box_rows), 1};
   const cuuint32_t estr[3] = {1, 1, 1};
   CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims,
                    strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,

@@ -51,6 +51,22 @@ int launch_attn_fwd_bf16_split_noalloc(const AttnArgs& a, const SplitPlan& sp, c
 // swizzle, rows past N of a slice read as zero.  False (and a message) on failure.
 bool encode_bf16_map(CUtensorMap* map, const void* base, int64_t BH, int64_t N, int64_t d,
                      char* msg, size_t msglen);
+// Same with a box of box_rows rows (64 columns, 128-byte swizzle).
+bool encode_bf16_map_box(CUtensorMap* map, const void* base, int64_t BH, int64_t N, int64_t d,
+                         int box_rows, char* msg, size_t msglen);
+
+// Validated arguments of one projection call (see include/moa_attn.h, moa_qkv_proj).
+struct ProjArgs {
+  const void* X;  // [B, N, d]
+  const void* W;  // [d, 2*H*dk + H*dv]
+  void* Q;
+  void* K;
+  void* V;
+  int64_t B, N, d, H, dk, dv;
+  cudaStream_t stream;
+};
+int launch_qkv_proj_bf16(const ProjArgs& a, char* msg, size_t msglen);
+cudaError_t proj_read_and_clear_status(unsigned* value);
 
 // Validated arguments of one backward call (see include/moa_attn.h, moa_attn_bwd).
 struct BwdArgs {

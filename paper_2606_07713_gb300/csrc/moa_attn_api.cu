@@ -283,18 +283,61 @@ int moa_attn_bwd(const void* Q, const void* K, const void* V, const void* O, con
   return MOA_OK;
 }
 
+int moa_qkv_proj(const void* X, const void* W, void* Q, void* K, void* V, int64_t B, int64_t N,
+                 int64_t d_model, int64_t H, int64_t d_k, int64_t d_v, int dtype, void* stream) {
+  if (!X || !W || !Q || !K || !V) return moa::fail(MOA_ERR_INVALID_ARG, "null tensor pointer");
+  if (B <= 0 || N <= 0 || d_model <= 0 || H <= 0 || d_k <= 0 || d_v <= 0)
+    return moa::fail(MOA_ERR_INVALID_ARG, "sizes must be >= 1");
+  if (dtype != MOA_BF16)
+    return moa::fail(MOA_ERR_UNSUPPORTED_DTYPE, "the projection takes bf16 tensors only (dtype %d)",
+                     dtype);
+  if ((d_k != 64 && d_k != 128) || (d_v != 64 && d_v != 128))
+    return moa::fail(MOA_ERR_UNSUPPORTED_SHAPE, "d_k, d_v must be 64 or 128; got %lld, %lld",
+                     (long long)d_k, (long long)d_v);
+  if (d_model % 8 != 0)
+    return moa::fail(MOA_ERR_MISALIGNED, "d_model must be a multiple of 8 (16-byte rows)");
+  const int64_t ncol = 2 * H * d_k + H * d_v;
+  const int64_t nx = moa::numel4(B, N, d_model, 1), nw = moa::numel4(d_model, ncol, 1, 1);
+  const int64_t nq = moa::numel4(B, H, N, d_k), nv = moa::numel4(B, H, N, d_v);
+  if (nx < 0 || nw < 0 || nq < 0 || nv < 0 || nx > INT64_MAX / 4 || nw > INT64_MAX / 4 ||
+      nq > INT64_MAX / 4 || nv > INT64_MAX / 4)
+    return moa::fail(MOA_ERR_UNSUPPORTED_SHAPE, "tensor sizes overflow 64-bit byte counts");
+  if (B * N > 0x7fffffffLL || ncol > 0x7fffffffLL || d_model > 0x7fffffffLL)
+    return moa::fail(MOA_ERR_UNSUPPORTED_SHAPE, "B*N, d_model and 2*H*d_k + H*d_v must be below 2^31");
+  const void* ptrs[5] = {X, W, Q, K, V};
+  for (const void* p : ptrs)
+    if (reinterpret_cast<uintptr_t>(p) % 16 != 0)
+      return moa::fail(MOA_ERR_MISALIGNED, "tensor pointer %p is not 16-byte aligned", p);
+  const void* out[3] = {Q, K, V};
+  const int64_t osz[3] = {nq * 2, nq * 2, nv * 2};
+  for (int i = 0; i < 3; ++i) {
+    if (moa::overlaps(out[i], osz[i], X, nx * 2) || moa::overlaps(out[i], osz[i], W, nw * 2))
+      return moa::fail(MOA_ERR_INVALID_ARG, "an output overlaps X or W");
+    for (int j = i + 1; j < 3; ++j)
+      if (moa::overlaps(out[i], osz[i], out[j], osz[j]))
+        return moa::fail(MOA_ERR_INVALID_ARG, "Q, K and V overlap");
+  }
+  moa::ProjArgs a{X, W, Q, K, V, B, N, d_model, H, d_k, d_v, static_cast<cudaStream_t>(stream)};
+  char msg[256] = {0};
+  const int rc = moa::launch_qkv_proj_bf16(a, msg, sizeof(msg));
+  if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
+  moa::t_last_error[0] = '\0';
+  return MOA_OK;
+}
+
 const char* moa_last_error(void) { return moa::t_last_error; }
 
 int moa_get_device_status(void* stream) {
   cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess)
     return moa::fail(MOA_ERR_CUDA, "stream synchronize: %s", cudaGetErrorString(e));
-  unsigned v = 0, vb = 0;
+  unsigned v = 0, vb = 0, vp = 0;
   e = moa::bf16_read_and_clear_status(&v);
   if (e == cudaSuccess) e = moa::bwd_read_and_clear_status(&vb);
+  if (e == cudaSuccess) e = moa::proj_read_and_clear_status(&vp);
   if (e != cudaSuccess)
     return moa::fail(MOA_ERR_CUDA, "status word read: %s", cudaGetErrorString(e));
-  v |= vb;
+  v |= vb | vp;
   if (v != 0)
     return moa::fail(MOA_ERR_DEVICE_TIMEOUT, "a kernel wait ran out (status %u)", v);
   return MOA_OK;

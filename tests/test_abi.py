@@ -161,3 +161,26 @@ def test_bwd_validation_without_gpu(L):
     assert call(q) == _lib.MOA_ERR_INVALID_ARG                          # dV aliases dQ
     q = list(P); q[9] = P[4]
     assert call(q) == _lib.MOA_ERR_INVALID_ARG                          # workspace aliases dO
+
+
+def test_qkv_proj_validation_without_gpu(L):
+    f = _lib.moa_qkv_proj
+    P = [0x1000000 * (i + 1) for i in range(5)]   # X, W, Q, K, V
+    ok = (2, 256, 512, 4, 64, 64)
+
+    def call(p=None, dims=ok, dtype=1):
+        return f(*(P if p is None else p), *dims, dtype, None)
+
+    for i in range(5):
+        q = list(P); q[i] = None
+        assert call(q) == _lib.MOA_ERR_INVALID_ARG
+    assert call(dtype=0) == _lib.MOA_ERR_UNSUPPORTED_DTYPE
+    assert call(dims=(2, 256, 512, 4, 96, 64)) == _lib.MOA_ERR_UNSUPPORTED_SHAPE
+    assert call(dims=(2, 256, 500, 4, 64, 64)) == _lib.MOA_ERR_MISALIGNED   # d_model % 8
+    assert call(dims=(0, 256, 512, 4, 64, 64)) == _lib.MOA_ERR_INVALID_ARG
+    q = list(P); q[3] = P[3] + 8
+    assert call(q) == _lib.MOA_ERR_MISALIGNED
+    q = list(P); q[2] = P[0]
+    assert call(q) == _lib.MOA_ERR_INVALID_ARG                            # Q aliases X
+    q = list(P); q[4] = P[3] + 64
+    assert call(q) == _lib.MOA_ERR_INVALID_ARG                            # V inside K
