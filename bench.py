@@ -5,7 +5,7 @@ N(0,1) from the seeded generator, scale=1/sqrt(d_k), no mask.  One step = one at
 forward over that batch (the whole hot path: one kernel launch).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference|classical]
-                    [--workload ID] [--shape B,H,N_q,N_k,d_k,d_v] [--pass fwd|bwd]
+                    [--workload ID] [--shape B,H,N_q,N_k,d_k,d_v] [--pass fwd|bwd|qkv]
 
 Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s: FLOPs of every step on every
 rank divided by the slowest rank's summed kernel time, measured with CUDA events on the
@@ -17,7 +17,9 @@ M_classical models (Section 8.2): the score matrix, its max-shifted exponentials
 normalised weights each materialised in device memory by eager PyTorch ops (cuBLAS GEMMs and
 elementwise/reduction kernels) -- a measurement of the comparison, not part of the library.
 `--shape` replaces the workload's sizes (bf16, same generator) for traffic sweeps.  `--pass bwd`
-times moa_attn_bwd (three launches) on the same workload instead of the forward pass.  Multi-GPU (torchrun): every rank runs its own full copy of the workload (the
+times moa_attn_bwd (three launches) on the same workload instead of the forward pass, and
+`--pass qkv` the fused projection moa_qkv_proj producing that workload's Q, K, V from an input
+X [B, N, H*d_k].  Multi-GPU (torchrun): every rank runs its own full copy of the workload (the
 (b, h) problems are independent; no collective on the data path), so scaling is weak.
 """
 from __future__ import annotations
@@ -45,7 +47,7 @@ DEFAULT_WORKLOAD = 2
 PROFILES = {2: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b4h16n2048d64.txt"),
             3: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b2h32n8192d128.txt")}
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2606_07713_gb300", "csrc", f)
-                  for f in ("attn_fwd_bf16_tc.cu", "ptx.cuh")]
+                  for f in ("attn_fwd_bf16_tc.cu", "ptx.cuh", "tc_common.cuh")]
 FLUSH_BYTES = 256 << 20
 
 
@@ -458,6 +460,149 @@ def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
 
 
 # ------------------------------------------------------------------------------------------
+# the fused input projection (--pass qkv)
+# ------------------------------------------------------------------------------------------
+def proj_inputs(cfg: I.AttnConfig):
+    """X [B, N, H*d_k] ~ N(0,1) and W [H*d_k, 2*H*d_k + H*d_v] ~ N(0,1)/sqrt(H*d_k) (bf16), from
+    the seeded generator (streams 5 and 6), so that Q, K, V have unit scale."""
+    s = cfg.shape
+    dm = s.H * s.d_k
+    ncol = 2 * s.H * s.d_k + s.H * s.d_v
+    x64 = I.normal(cfg.the_seed, 5, s.B * s.N_q * dm)
+    w64 = I.normal(cfg.the_seed, 6, dm * ncol) / math.sqrt(dm)
+    xb = I.f32_to_bf16_bits(x64.astype(np.float32)).reshape(s.B, s.N_q, dm)
+    wb = I.f32_to_bf16_bits(w64.astype(np.float32)).reshape(dm, ncol)
+    return xb, wb
+
+
+def run_ours_qkv(args, cfg: I.AttnConfig) -> None:
+    import torch
+    import torch.distributed as dist
+
+    import paper_2606_07713_gb300 as pkg
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    pkg.lib()
+    s = cfg.shape
+    if cfg.dtype != "bf16" or s.N_q != s.N_k:
+        raise SystemExit("the projection pass takes bf16 self-attention workloads (N_q = N_k)")
+    xb, wb = proj_inputs(cfg)
+    x, w = (to_device_bf16(b, dev) for b in (xb, wb))
+    hx, hw = (torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).view(torch.bfloat16)
+              .pin_memory() for b in (xb, wb))
+    q = torch.empty((s.B, s.H, s.N_q, s.d_k), dtype=torch.bfloat16, device=dev)
+    k = torch.empty_like(q)
+    v = torch.empty((s.B, s.H, s.N_q, s.d_v), dtype=torch.bfloat16, device=dev)
+    hout = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in (q, k, v)]
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    dm = s.H * s.d_k
+    ncol = 2 * s.H * s.d_k + s.H * s.d_v
+    flops = 2.0 * s.B * s.N_q * dm * ncol
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        pkg.qkv_proj(x, w, s.H, s.d_k, s.d_v, out=(q, k, v))
+    torch.cuda.synchronize(dev)
+    pkg.check(pkg.get_device_status())
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    barrier()
+    for i in range(args.steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        pkg.qkv_proj(x, w, s.H, s.d_k, s.d_v, out=(q, k, v), stream=stream)
+        ev[i][1].record(stream)
+    barrier()
+    kern_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = float(np.sum(kern_ms))
+    ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    barrier()
+    for i in range(args.steps):
+        flush.zero_()
+        ev2[i][0].record(stream)
+        x.copy_(hx, non_blocking=True)
+        w.copy_(hw, non_blocking=True)
+        pkg.qkv_proj(x, w, s.H, s.d_k, s.d_v, out=(q, k, v), stream=stream)
+        for h_, d_ in zip(hout, (q, k, v)):
+            h_.copy_(d_, non_blocking=True)
+        ev2[i][1].record(stream)
+    barrier()
+    clocks = sampler.stop()
+    e2e_ms = float(np.sum([a.elapsed_time(b) for a, b in ev2]))
+    pkg.check(pkg.get_device_status())
+    total_ms, e2e_ms = reduce_max_over_ranks([total_ms, e2e_ms], device=dev)
+    if rank == 0:
+        peaks, peak_src = measured_peaks()
+        achieved = flops / (float(np.mean(kern_ms)) * 1e-3) / 1e12
+        peak = float(peaks["bf16_tflops"])
+        line = {
+            "metric": "fused QKV projection TFLOP/s and % of GB300 bf16 peak",
+            "value": round(whole_job_tflops(flops, args.steps, world, total_ms), 2),
+            "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(total_ms / args.steps, 6), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic: seeded X ~ N(0,1), W ~ N(0,1)/sqrt(d_model)",
+            "config": {"workload": f"bf16 QKV projection, X [{s.B}, {s.N_q}, {dm}] x W [{dm}, {ncol}]"
+                                   f" -> Q, K [{s.B}, {s.H}, {s.N_q}, {s.d_k}], V [.., {s.d_v}]",
+                       "B": s.B, "N": s.N_q, "d_model": dm, "H": s.H, "d_k": s.d_k, "d_v": s.d_v,
+                       "l2": f"flushed before every step ({FLUSH_BYTES >> 20} MiB write, untimed)",
+                       "pass": "projection (moa_qkv_proj)"},
+            "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": peak,
+                         "peak_source": f"{peak_src} bf16_tflops (burst; kernel timed alone)",
+                         "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": None,
+                         "kernel": "qkv_proj_bf16_tc_kernel"},
+            "e2e": {"value": round(whole_job_tflops(flops, args.steps, world, e2e_ms), 2),
+                    "unit": "TFLOP/s",
+                    "h2d_bytes_per_step": int(hx.numel() * 2 + hw.numel() * 2),
+                    "d2h_bytes_per_step": int(sum(t.numel() * 2 for t in hout)),
+                    "api": "qkv_proj with host copies of X, W and Q, K, V"},
+            "gpu_launches": args.steps,
+            "clocks": clocks,
+        }
+        if world == 1:
+            line["cpu_baseline"] = cpu_baseline_qkv(cfg, xb, wb, budget_s=args.cpu_budget)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def cpu_baseline_qkv(cfg, xb, wb, budget_s: float = 12.0) -> dict:
+    import oracle
+    orc = oracle.get()
+    s = cfg.shape
+    x = I.bf16_bits_to_f32(xb)
+    w = I.bf16_bits_to_f32(wb)
+    dm, ncol = w.shape
+    n = min(s.N_q, 64)
+    t0 = time.perf_counter()
+    orc.qkv_proj(x[:1, :n], w, s.H, s.d_k, s.d_v)
+    dt = time.perf_counter() - t0
+    n2 = int(min(s.N_q, max(n, n * budget_s / max(dt, 1e-6) / 2)))
+    t0 = time.perf_counter()
+    orc.qkv_proj(x[:1, :n2], w, s.H, s.d_k, s.d_v)
+    dt = time.perf_counter() - t0
+    return {"value": round(2.0 * n2 * dm * ncol / dt / 1e12, 6), "unit": "TFLOP/s",
+            "cores": orc.max_threads(), "kind": "oracle",
+            "sample": f"{n2} of {s.B * s.N_q} tokens, fp64, {dt:.1f} s"}
+
+
+# ------------------------------------------------------------------------------------------
 # the classical path (what Eq. M_classical counts), for the measured traffic comparison
 # ------------------------------------------------------------------------------------------
 def classical_step(q, k, v, scale):
@@ -615,8 +760,8 @@ def main():
     ap.add_argument("--workload", type=int, default=DEFAULT_WORKLOAD, choices=sorted(I.CONFIGS))
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle time for the cpu_baseline sample")
-    ap.add_argument("--pass", dest="which", choices=["fwd", "bwd"], default="fwd",
-                    help="time the forward (default) or the backward pass")
+    ap.add_argument("--pass", dest="which", choices=["fwd", "bwd", "qkv"], default="fwd",
+                    help="time the forward (default), the backward pass or the QKV projection")
     ap.add_argument("--shape", default=None,
                     help="B,H,N_q,N_k,d_k,d_v: a bf16 workload of this shape instead of --workload")
     args = ap.parse_args()
@@ -634,6 +779,8 @@ def main():
         run_classical(args, cfg)
     elif args.which == "bwd":
         run_ours_bwd(args, cfg)
+    elif args.which == "qkv":
+        run_ours_qkv(args, cfg)
     else:
         run_ours(args, cfg)
 
