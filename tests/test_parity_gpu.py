@@ -81,3 +81,20 @@ def test_bf16_unusual_scales(oracle, scale):
     x = I.make_inputs(cfg)
     o = run(x, scale)
     assert_close(o, oracle.attn(x.q, x.k, x.v, scale), "bf16", f"scale={scale}")
+
+
+@pytest.mark.parametrize("dk,dv", [(64, 64), (128, 64)])
+def test_bf16_grid_beyond_one_wave(oracle, dk, dv):
+    """More 256-row work items than SMs (a second, nearly empty wave).  Every row of every head
+    is checked, including rows of a half-valid second tile (N_q = 200) and the LSE output."""
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    H = n_sm + 10                       # n_sm + 10 work items
+    cfg = I.custom_config(1, H, 200, 300, dk, dv, dtype="bf16", seed=H + dk)
+    x = I.make_inputs(cfg)
+    q, k, v = to_device(x)
+    o, lse = pkg.attn_fwd_lse(q, k, v, x.scale)
+    torch.cuda.synchronize()
+    pkg.check(pkg.get_device_status())
+    ref, lref = oracle.attn_lse(x.q, x.k, x.v, x.scale)
+    assert_close(o.float().cpu().numpy(), ref, "bf16", f"tail d_k={dk} d_v={dv}")
+    assert np.max(np.abs(lse.double().cpu().numpy() - lref)) <= 1e-3 * (1 + np.max(np.abs(lref)))

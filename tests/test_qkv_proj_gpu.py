@@ -99,3 +99,22 @@ def test_qkv_proj_feeds_attention(oracle):
         assert rel_err(a, b) <= 1e-2
     ref = oracle.attn(qb, kb, vb, 1.0 / np.sqrt(dk))
     assert rel_err(o.float().cpu().numpy(), ref) <= 2e-2
+
+
+@pytest.mark.parametrize("shape", [(1, 12800, 128, 2, 64, 64), (4, 2048, 256, 16, 64, 64)],
+                         ids=["many-token-tiles", "bench-like"])
+def test_qkv_proj_large_grids(oracle, shape):
+    """Grids of several tiles per persistent CTA (both accumulators reused many times), checked
+    on the first 300 tokens of every batch entry (each token's outputs depend on that token's
+    row of X only)."""
+    B, N, d, H, dk, dv = shape
+    r = np.random.default_rng(sum(shape))
+    xf = r.normal(size=(B, N, d))
+    wf = r.normal(size=(d, 2 * H * dk + H * dv)) / np.sqrt(d)
+    x32, w32, got = run(xf, wf, H, dk, dv)
+    n = min(N, 300)
+    ref = oracle.qkv_proj(np.ascontiguousarray(x32[:, :n]), w32, H, dk, dv)
+    for name, a, b in zip("QKV", got, ref):
+        err = rel_err(a[:, :, :n], b)
+        assert err <= 1e-2, f"{shape} {name}: {err:.3e}"
+        assert np.all(np.isfinite(a))
