@@ -286,20 +286,9 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
       const uint32_t tDV = tmem + C::kTmemDV, tDK = tmem + C::kTmemDK;
       int slot = 0;
       uint32_t phase = 0;
-      bool ok = wait_bounded(kv_full, 0, wc);
-      for (int i = 0; ok && i < n_qb; ++i) {
-        const int st = slot;
-        ok = wait_bounded(full_bar(slot), phase, wc);
-        if (++slot == C::kStages) {
-          slot = 0;
-          phase ^= 1u;
-        }
-        if (!ok) break;
-        tc_fence_after_sync();
-        const uint32_t sQ = sStage + st * C::kStageBytes, sDO = sQ + C::kQBytes;
-        const uint32_t par = uint32_t(i) & 1u;
-        // S^T = K Q^T: M = 128 keys, N = 128 queries, both operands K-major (d_k contiguous);
-        // reduction step kk is panel kk/4, 32 bytes further per step inside it.
+      // S^T = K Q^T: M = 128 keys, N = 128 queries, both operands K-major (d_k contiguous);
+      // reduction step kk is panel kk/4, 32 bytes further per step inside it.
+      auto issue_s = [&](uint32_t sQ) {
 #pragma unroll
         for (int kk = 0; kk < DK / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
@@ -307,7 +296,9 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
                      kIdescS, kk > 0 ? 1u : 0u);
         }
         mma_commit(s_full);
-        // dP^T = V dO^T: M = 128 keys, N = 128 queries, reduction over d_v.
+      };
+      // dP^T = V dO^T: M = 128 keys, N = 128 queries, reduction over d_v.
+      auto issue_dp = [&](uint32_t sDO) {
 #pragma unroll
         for (int kk = 0; kk < DV / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
@@ -315,6 +306,27 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
                      kIdescS, kk > 0 ? 1u : 0u);
         }
         mma_commit(dp_full);
+      };
+      auto stage = [&](int st) { return sStage + st * C::kStageBytes; };
+      // Issue order S(0) dP(0) | dV(0) S(1) dK(0) dP(1) | dV(1) S(2) dK(1) dP(2) | ...: the scores
+      // of block i+1 are ready when the compute warps finish dS of block i, and the tensor pipe
+      // works on dK(i) and dP(i+1) while they form P(i+1).  S(i+1) overwrites the columns of
+      // P^T(i) only after dV(i), and dP(i+1) those of dS^T(i) only after dK(i), both issued
+      // earlier (tensor-core operations of one CTA complete in issue order).
+      bool ok = wait_bounded(kv_full, 0, wc) && wait_bounded(full_bar(0), 0, wc);
+      if (ok) {
+        tc_fence_after_sync();
+        issue_s(stage(0));
+        issue_dp(stage(0) + C::kQBytes);
+      }
+      for (int i = 0; ok && i < n_qb; ++i) {
+        const int st = slot;
+        if (++slot == C::kStages) {
+          slot = 0;
+          phase ^= 1u;
+        }
+        const uint32_t sQ = stage(st), sDO = sQ + C::kQBytes;
+        const uint32_t par = uint32_t(i) & 1u;
         // dV += P^T dO: A = P^T (bf16, TMEM), B = dO tile MN-major (d_v contiguous): groups of 8
         // query rows 1024 B apart, 64-column panels kPanelBytes apart.
         ok = wait_bounded(p_ready, par, wc);
@@ -325,6 +337,13 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
           mma_f16_ts(tDV, tS + half_split_col(kk),
                      make_sdesc_sw128(sDO + kk * 2048, kPanelBytes, 1024), kIdescDV,
                      (kk > 0 || i > 0) ? 1u : 0u);
+        const bool more = i + 1 < n_qb;
+        if (more) {
+          ok = wait_bounded(full_bar(slot), phase, wc);
+          if (!ok) break;
+          tc_fence_after_sync();
+          issue_s(stage(slot));
+        }
         // dK += dS^T Q (scale applied in the epilogue): B = Q tile MN-major.
         ok = wait_bounded(ds_ready, par, wc);
         if (!ok) break;
@@ -335,6 +354,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
                      make_sdesc_sw128(sQ + kk * 2048, kPanelBytes, 1024), kIdescDK,
                      (kk > 0 || i > 0) ? 1u : 0u);
         mma_commit(empty_bar(st));
+        if (more) issue_dp(stage(slot) + C::kQBytes);
       }
       // Always signal once everything issued has completed, so that TMEM is quiescent before
       // it is freed even on the abort path.
@@ -445,8 +465,8 @@ struct DqCfg {
   static constexpr int kOffQ = 0;
   static constexpr int kOffDO = kQBytes;
   static constexpr int kOffStage = kQBytes + kDOBytes;
-  // barriers: full[NS], empty[NS], q_full, s_full, dp_full, ds_ready, acc_done
-  static constexpr int kNumBars = 2 * kStages + 5;
+  // barriers: full[NS], empty[NS], q_full, s_full, dp_full, ds_ready, acc_done, s_free
+  static constexpr int kNumBars = 2 * kStages + 6;
   static constexpr int kOffBar = kOffStage + kStages * kStageBytes;
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;
   static constexpr int kSmemBytes = kOffMisc + 16 + 1024;
@@ -474,7 +494,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
   auto empty_bar = [&](int s) { return bar0 + 8u * (C::kStages + s); };
   const uint32_t q_full = bar0 + 8u * (2 * C::kStages);
   const uint32_t s_full = q_full + 8, dp_full = q_full + 16, ds_ready = q_full + 24;
-  const uint32_t acc_done = q_full + 32;
+  const uint32_t acc_done = q_full + 32, s_free = q_full + 40;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
 
@@ -495,6 +515,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     mbar_init(dp_full, 1);
     mbar_init(ds_ready, 8 * 32);
     mbar_init(acc_done, 1);
+    mbar_init(s_free, 8 * 32);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -560,18 +581,9 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
       const uint32_t tS = tmem + C::kTmemS, tDP = tmem + C::kTmemDP, tDQ = tmem + C::kTmemDQ;
       int slot = 0;
       uint32_t phase = 0;
-      bool ok = wait_bounded(q_full, 0, wc);
-      for (int j = 0; ok && j < n_kb; ++j) {
-        const int st = slot;
-        ok = wait_bounded(full_bar(slot), phase, wc);
-        if (++slot == C::kStages) {
-          slot = 0;
-          phase ^= 1u;
-        }
-        if (!ok) break;
-        tc_fence_after_sync();
-        const uint32_t sK = sStage + st * C::kStageBytes, sV = sK + C::kKBytes;
-        // S = Q K^T (M = 128 queries, N = 128 keys, K-major operands)
+      auto stage = [&](int st) { return sStage + st * C::kStageBytes; };
+      // S = Q K^T (M = 128 queries, N = 128 keys, K-major operands)
+      auto issue_s = [&](uint32_t sK) {
 #pragma unroll
         for (int kk = 0; kk < DK / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
@@ -579,7 +591,9 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                      kIdescS, kk > 0 ? 1u : 0u);
         }
         mma_commit(s_full);
-        // dP = dO V^T (reduction over d_v)
+      };
+      // dP = dO V^T (reduction over d_v)
+      auto issue_dp = [&](uint32_t sV) {
 #pragma unroll
         for (int kk = 0; kk < DV / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
@@ -587,16 +601,42 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
                      kIdescS, kk > 0 ? 1u : 0u);
         }
         mma_commit(dp_full);
+      };
+      // Issue order S(0) dP(0) | S(1) dQ(0) dP(1) | S(2) dQ(1) dP(2) | ...: S(j+1) goes as soon as
+      // the compute warps hold S(j) in registers (s_free), so they find it ready after dS(j);
+      // dP(j+1) overwrites the columns of dS(j) only after dQ(j), issued earlier.
+      bool ok = wait_bounded(q_full, 0, wc) && wait_bounded(full_bar(0), 0, wc);
+      if (ok) {
+        tc_fence_after_sync();
+        issue_s(stage(0));
+        issue_dp(stage(0) + C::kKBytes);
+      }
+      for (int j = 0; ok && j < n_kb; ++j) {
+        const int st = slot;
+        if (++slot == C::kStages) {
+          slot = 0;
+          phase ^= 1u;
+        }
+        const uint32_t par = uint32_t(j) & 1u;
+        const bool more = j + 1 < n_kb;
+        if (more) {
+          ok = wait_bounded(full_bar(slot), phase, wc) && wait_bounded(s_free, par, wc);
+          if (!ok) break;
+          tc_fence_after_sync();
+          issue_s(stage(slot));
+        }
         // dQ += dS K (scale applied in the epilogue): A = dS (bf16, TMEM), B = K tile MN-major.
-        ok = wait_bounded(ds_ready, uint32_t(j) & 1u, wc);
+        ok = wait_bounded(ds_ready, par, wc);
         if (!ok) break;
         tc_fence_after_sync();
+        const uint32_t sK = stage(st);
 #pragma unroll
         for (int kk = 0; kk < kBlk / 16; ++kk)
           mma_f16_ts(tDQ, tDP + half_split_col(kk),
                      make_sdesc_sw128(sK + kk * 2048, kPanelBytes, 1024), kIdescDQ,
                      (kk > 0 || j > 0) ? 1u : 0u);
         mma_commit(empty_bar(st));
+        if (more) issue_dp(stage(slot) + C::kKBytes);
       }
       mma_commit(acc_done);
     }
@@ -620,6 +660,9 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
       tc_fence_after_sync();
       uint32_t r[64];
       tmem_load_row64(tS, r);
+      // S(j) is in registers: the issuer may write S(j+1) over it
+      tc_fence_before_sync();
+      mbar_arrive(s_free);
       float p[64];
 #pragma unroll
       for (int k = 0; k < 64; k += 2) {
