@@ -24,12 +24,13 @@
 // pair instead of 5.
 //
 // CTA organisation of both tile kernels (one CTA per SM: 512 TMEM columns):
-//   warps 0-7: 128 rows x 2 column halves.  Warp w owns TMEM lanes 32*(w%4).. (its rows) and
-//              columns [64*(w/4), +64) of the 128-wide score tiles; it writes its bf16 P or dS
-//              back into the first 32 of those columns, so the two halves never overlap.  The
-//              products that read them take K-steps 0-3 from columns 0-31 and 4-7 from 64-95.
-//   warp 8:    TMEM allocation and the single thread that issues every tcgen05.mma;
-//   warp 9:    the single thread that issues every TMA copy.
+//   warps 0..4P-1: 128 rows x P column parts (P = 4 for d_k + d_v = 128, else 2).  Warp w owns
+//              TMEM lanes 32*(w%4).. (its rows) and columns [(128/P)*(w/4), +128/P) of the
+//              128-wide score tiles; it writes its bf16 P or dS back into the first half of those
+//              columns, so the parts never overwrite each other's unread values (part_col gives
+//              the products' operand columns).
+//   warp 4P:   TMEM allocation and the single thread that issues every tcgen05.mma;
+//   warp 4P+1: the single thread that issues every TMA copy.
 // Every mbarrier wait is bounded; on expiry the kernel records MOA_ERR_DEVICE_TIMEOUT in
 // g_moa_bwd_status, every role leaves its loop, and TMEM is still freed.
 #include <cuda.h>
@@ -54,9 +55,21 @@ using namespace ptx;
 using namespace tc;
 
 constexpr int kBlk = 128;          // rows of every tile (= TMEM lanes) and keys per key block
-constexpr int kThreads = 320;      // 8 compute warps, MMA warp, TMA warp
-constexpr int kMmaWarp = 8;        // also allocates and frees TMEM
-constexpr int kLoadWarp = 9;
+
+// Compute-warp layout: P parts of the 128-wide tiles per TMEM lane quarter, 4P compute warps,
+// then the MMA warp and the TMA warp.  P = 4 (four warps per scheduler) where the tile products
+// are short (d_k + d_v = 128) and the exponentials dominate; P = 2 otherwise.
+template <int P>
+struct Warps {
+  static constexpr int kParts = P;
+  static constexpr int kCols = kBlk / P;             // fp32 columns per compute thread
+  static constexpr int kComputeWarps = 4 * P;
+  static constexpr int kComputeThreads = 32 * kComputeWarps;
+  static constexpr int kThreads = kComputeThreads + 64;
+  static constexpr int kMmaWarp = kComputeWarps;     // also allocates and frees TMEM
+  static constexpr int kLoadWarp = kComputeWarps + 1;
+};
+__host__ __device__ constexpr int bwd_parts(int dk, int dv) { return dk + dv <= 128 ? 4 : 2; }
 constexpr int kTmemCols = 512;
 constexpr int kPanelBytes = 128 * 128;  // one 128-byte-swizzle panel: 64 bf16 columns x 128 rows
 constexpr int kVecBytes = kBlk * 4;     // 128 fp32 per-row values
@@ -66,19 +79,31 @@ __host__ __device__ constexpr int ring_stages(int dk, int dv) {
   return dk + dv <= 128 ? 4 : (dk + dv <= 192 ? 3 : 2);
 }
 
-// TMEM column of K-step kk (16 rows of the reduction axis) of a bf16 operand written by the two
-// column halves: steps 0-3 from columns 0-31, steps 4-7 from columns 64-95.
-__device__ __forceinline__ uint32_t half_split_col(int kk) {
-  return kk < 4 ? uint32_t(kk * 8) : uint32_t(64 + (kk - 4) * 8);
+// TMEM column of K-step kk (16 rows of the reduction axis) of a bf16 operand written by the
+// column parts: part p packs its COLS values into the first COLS/2 columns of its own range
+// [p*COLS, +COLS), so the 16 rows of step kk sit at column (16kk/COLS)*COLS + (16kk%COLS)/2.
+template <int COLS>
+__device__ __forceinline__ uint32_t part_col(int kk) {
+  return uint32_t((kk * 16 / COLS) * COLS + (kk * 16 % COLS) / 2);
 }
 
-// Loads 64 fp32 TMEM columns of this thread's lane (two x32 loads) and waits.
-__device__ __forceinline__ void tmem_load_row64(uint32_t taddr, uint32_t* r) {
-  tmem_ld_32x32b_x32(taddr, r);
-  tmem_ld_32x32b_x32(taddr + 32, r + 32);
+// Loads COLS fp32 TMEM columns of this thread's lane and waits.
+template <int COLS>
+__device__ __forceinline__ void tmem_load_part(uint32_t taddr, uint32_t* r) {
+#pragma unroll
+  for (int c = 0; c < COLS; c += 32) tmem_ld_32x32b_x32(taddr + c, r + c);
   tmem_wait_ld();
-  reg_anchor_x32(r);
-  reg_anchor_x32(r + 32);
+#pragma unroll
+  for (int c = 0; c < COLS; c += 32) reg_anchor_x32(r + c);
+}
+
+// Stores COLS/2 packed bf16 pairs to this thread's lane.
+template <int COLS>
+__device__ __forceinline__ void tmem_store_part(uint32_t taddr, const uint32_t* pk) {
+  if constexpr (COLS == 64)
+    tmem_st_32x32b_x32(taddr, pk);
+  else
+    tmem_st_32x32b_x16(taddr, pk);
 }
 
 // Writes ncols fp32 TMEM columns of this thread's lane, times mul, as bf16 to dst (16-B aligned).
@@ -152,7 +177,7 @@ attn_bwd_pre_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfloat16* __
 // dK and dV: one CTA per (b, h, 128-key block)
 // ------------------------------------------------------------------------------------------
 template <int DK, int DV>
-struct DkDvCfg {
+struct DkDvCfg : Warps<bwd_parts(DK, DV)> {
   static_assert((DK == 64 || DK == 128) && (DV == 64 || DV == 128), "d_k, d_v in {64, 128}");
   static constexpr int kKBytes = kBlk * DK * 2;
   static constexpr int kVBytes = kBlk * DV * 2;
@@ -176,13 +201,15 @@ struct DkDvCfg {
 };
 
 template <int DK, int DV>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(DkDvCfg<DK, DV>::kThreads, 1)
 attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                      const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmDO,
                      const float* __restrict__ nL, const float* __restrict__ Dd,
                      __nv_bfloat16* __restrict__ dK, __nv_bfloat16* __restrict__ dV, int Nk,
                      int Nq_pad, int n_kblocks, float c_log2, float scale, uint64_t wait_limit_ns) {
   using C = DkDvCfg<DK, DV>;
+  constexpr int kParts = C::kParts, kCols = C::kCols, kComputeThreads = C::kComputeThreads;
+  constexpr int kMmaWarp = C::kMmaWarp, kLoadWarp = C::kLoadWarp;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -213,8 +240,8 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
     mbar_init(kv_full, 1);
     mbar_init(s_full, 1);
     mbar_init(dp_full, 1);
-    mbar_init(p_ready, 8 * 32);
-    mbar_init(ds_ready, 8 * 32);
+    mbar_init(p_ready, kComputeThreads);
+    mbar_init(ds_ready, kComputeThreads);
     mbar_init(acc_done, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -334,7 +361,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
         tc_fence_after_sync();
 #pragma unroll
         for (int kk = 0; kk < kBlk / 16; ++kk)
-          mma_f16_ts(tDV, tS + half_split_col(kk),
+          mma_f16_ts(tDV, tS + part_col<kCols>(kk),
                      make_sdesc_sw128(sDO + kk * 2048, kPanelBytes, 1024), kIdescDV,
                      (kk > 0 || i > 0) ? 1u : 0u);
         const bool more = i + 1 < n_qb;
@@ -350,7 +377,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
         tc_fence_after_sync();
 #pragma unroll
         for (int kk = 0; kk < kBlk / 16; ++kk)
-          mma_f16_ts(tDK, tDP + half_split_col(kk),
+          mma_f16_ts(tDK, tDP + part_col<kCols>(kk),
                      make_sdesc_sw128(sQ + kk * 2048, kPanelBytes, 1024), kIdescDK,
                      (kk > 0 || i > 0) ? 1u : 0u);
         mma_commit(empty_bar(st));
@@ -362,12 +389,12 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
     }
   } else {
     // ---------------------------------------------------------------- compute warps
-    const int half = warp >> 2;              // column half of the 128-query tiles
+    const int part = warp >> 2;              // column part of the 128-query tiles
     const int lane_base = (warp & 3) * 32;   // TMEM lanes (key rows) of this warp
     const int row = lane_base + lane;        // key row inside the block
     const uint32_t lanes = uint32_t(lane_base) << 16;
-    const uint32_t tS = tmem + lanes + C::kTmemS + half * 64;
-    const uint32_t tDP = tmem + lanes + C::kTmemDP + half * 64;
+    const uint32_t tS = tmem + lanes + C::kTmemS + part * kCols;
+    const uint32_t tDP = tmem + lanes + C::kTmemDP + part * kCols;
     const uint64_t cc = pack_f32x2(c_log2, c_log2);
     int slot = 0;
     uint32_t phase = 0;
@@ -386,36 +413,36 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
       tc_fence_after_sync();
       const float* vec = reinterpret_cast<const float*>(smem + C::kOffStage + st * C::kStageBytes +
                                                         C::kQBytes + C::kDOBytes);
-      const float4* nl4 = reinterpret_cast<const float4*>(vec + half * 64);
-      const float4* d4 = reinterpret_cast<const float4*>(vec + kBlk + half * 64);
-      uint32_t r[64];
-      tmem_load_row64(tS, r);
-      float p[64];
+      const float4* nl4 = reinterpret_cast<const float4*>(vec + part * kCols);
+      const float4* d4 = reinterpret_cast<const float4*>(vec + kBlk + part * kCols);
+      uint32_t r[kCols];
+      tmem_load_part<kCols>(tS, r);
+      float p[kCols];
 #pragma unroll
-      for (int q = 0; q < 64; q += 4) {
+      for (int q = 0; q < kCols; q += 4) {
         const float4 l = nl4[q >> 2];
         ffma2(p[q], p[q + 1], __uint_as_float(r[q]), __uint_as_float(r[q + 1]), cc,
               pack_f32x2(l.x, l.y));
         ffma2(p[q + 2], p[q + 3], __uint_as_float(r[q + 2]), __uint_as_float(r[q + 3]), cc,
               pack_f32x2(l.z, l.w));
       }
-      uint32_t pk[32];
+      uint32_t pk[kCols / 2];
 #pragma unroll
-      for (int q = 0; q < 64; q += 2) {
+      for (int q = 0; q < kCols; q += 2) {
         p[q] = ex2_approx(p[q]);
         p[q + 1] = ex2_approx(p[q + 1]);
         pk[q >> 1] = pack_bf16x2(p[q], p[q + 1]);
       }
-      tmem_st_32x32b_x32(tS, pk);
+      tmem_store_part<kCols>(tS, pk);
       tmem_wait_st();
       tc_fence_before_sync();
       mbar_arrive(p_ready);
       ok = wait_bounded(dp_full, par, wc);
       if (!ok) break;
       tc_fence_after_sync();
-      tmem_load_row64(tDP, r);
+      tmem_load_part<kCols>(tDP, r);
 #pragma unroll
-      for (int q = 0; q < 64; q += 4) {
+      for (int q = 0; q < kCols; q += 4) {
         const float4 d = d4[q >> 2];
         const float s0 = p[q] * (__uint_as_float(r[q]) - d.x);
         const float s1 = p[q + 1] * (__uint_as_float(r[q + 1]) - d.y);
@@ -424,20 +451,27 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
         pk[q >> 1] = pack_bf16x2(s0, s1);
         pk[(q >> 1) + 1] = pack_bf16x2(s2, s3);
       }
-      tmem_st_32x32b_x32(tDP, pk);
+      tmem_store_part<kCols>(tDP, pk);
       tmem_wait_st();
       tc_fence_before_sync();
       mbar_arrive(ds_ready);
     }
-    // Epilogue: half 0 writes dV, half 1 writes scale * dK (rows past N_k are not stored).
+    // Epilogue: the first half of the parts write dV, the second half scale * dK, each part a
+    // slice of the columns (rows past N_k are not stored).
     if (ok && wait_bounded(acc_done, 0, wc)) {
       tc_fence_after_sync();
       const bool valid = k0 + row < Nk;
       const size_t grow = size_t(bh) * Nk + size_t(k0 + row);
-      if (half == 0)
-        store_row_bf16<DV>(tmem + lanes + C::kTmemDV, 1.0f, dV + grow * DV, valid);
-      else
-        store_row_bf16<DK>(tmem + lanes + C::kTmemDK, scale, dK + grow * DK, valid);
+      constexpr int kHalf = kParts / 2;
+      if (part < kHalf) {
+        constexpr int w = DV / kHalf;
+        store_row_bf16<w>(tmem + lanes + C::kTmemDV + part * w, 1.0f, dV + grow * DV + part * w,
+                          valid);
+      } else {
+        constexpr int w = DK / kHalf;
+        const int q = part - kHalf;
+        store_row_bf16<w>(tmem + lanes + C::kTmemDK + q * w, scale, dK + grow * DK + q * w, valid);
+      }
     }
   }
 
@@ -454,7 +488,7 @@ attn_bwd_dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_const
 // dQ: one CTA per (b, h, 128-row query block)
 // ------------------------------------------------------------------------------------------
 template <int DK, int DV>
-struct DqCfg {
+struct DqCfg : Warps<bwd_parts(DK, DV)> {
   static_assert((DK == 64 || DK == 128) && (DV == 64 || DV == 128), "d_k, d_v in {64, 128}");
   static constexpr int kQBytes = kBlk * DK * 2;
   static constexpr int kDOBytes = kBlk * DV * 2;
@@ -476,13 +510,15 @@ struct DqCfg {
 };
 
 template <int DK, int DV>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(DqCfg<DK, DV>::kThreads, 1)
 attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmDO,
                    const float* __restrict__ nL, const float* __restrict__ Dd,
                    __nv_bfloat16* __restrict__ dQ, int Nq, int Nk, int Nq_pad, int n_qblocks,
                    float c_log2, float scale, uint64_t wait_limit_ns) {
   using C = DqCfg<DK, DV>;
+  constexpr int kCols = C::kCols, kComputeThreads = C::kComputeThreads;
+  constexpr int kMmaWarp = C::kMmaWarp, kLoadWarp = C::kLoadWarp;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -513,9 +549,9 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     mbar_init(q_full, 1);
     mbar_init(s_full, 1);
     mbar_init(dp_full, 1);
-    mbar_init(ds_ready, 8 * 32);
+    mbar_init(ds_ready, kComputeThreads);
     mbar_init(acc_done, 1);
-    mbar_init(s_free, 8 * 32);
+    mbar_init(s_free, kComputeThreads);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -632,7 +668,7 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
         const uint32_t sK = stage(st);
 #pragma unroll
         for (int kk = 0; kk < kBlk / 16; ++kk)
-          mma_f16_ts(tDQ, tDP + half_split_col(kk),
+          mma_f16_ts(tDQ, tDP + part_col<kCols>(kk),
                      make_sdesc_sw128(sK + kk * 2048, kPanelBytes, 1024), kIdescDQ,
                      (kk > 0 || j > 0) ? 1u : 0u);
         mma_commit(empty_bar(st));
@@ -642,12 +678,12 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
     }
   } else {
     // ---------------------------------------------------------------- compute warps
-    const int half = warp >> 2;              // column half of the 128-key tiles
+    const int part = warp >> 2;              // column part of the 128-key tiles
     const int lane_base = (warp & 3) * 32;   // TMEM lanes (query rows) of this warp
     const int row = lane_base + lane;
     const uint32_t lanes = uint32_t(lane_base) << 16;
-    const uint32_t tS = tmem + lanes + C::kTmemS + half * 64;
-    const uint32_t tDP = tmem + lanes + C::kTmemDP + half * 64;
+    const uint32_t tS = tmem + lanes + C::kTmemS + part * kCols;
+    const uint32_t tDP = tmem + lanes + C::kTmemDP + part * kCols;
     const size_t vrow = size_t(bh) * Nq_pad + size_t(q0 + row);  // padded: always in range
     const float nl = nL[vrow], dd = Dd[vrow];
     const uint64_t cc = pack_f32x2(c_log2, c_log2);
@@ -658,14 +694,14 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
       ok = wait_bounded(s_full, par, wc);
       if (!ok) break;
       tc_fence_after_sync();
-      uint32_t r[64];
-      tmem_load_row64(tS, r);
+      uint32_t r[kCols];
+      tmem_load_part<kCols>(tS, r);
       // S(j) is in registers: the issuer may write S(j+1) over it
       tc_fence_before_sync();
       mbar_arrive(s_free);
-      float p[64];
+      float p[kCols];
 #pragma unroll
-      for (int k = 0; k < 64; k += 2) {
+      for (int k = 0; k < kCols; k += 2) {
         ffma2(p[k], p[k + 1], __uint_as_float(r[k]), __uint_as_float(r[k + 1]), cc, nn);
         p[k] = ex2_approx(p[k]);
         p[k + 1] = ex2_approx(p[k + 1]);
@@ -673,23 +709,25 @@ attn_bwd_dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constan
       ok = wait_bounded(dp_full, par, wc);
       if (!ok) break;
       tc_fence_after_sync();
-      tmem_load_row64(tDP, r);
-      uint32_t pk[32];
+      tmem_load_part<kCols>(tDP, r);
+      uint32_t pk[kCols / 2];
 #pragma unroll
-      for (int k = 0; k < 64; k += 2)
+      for (int k = 0; k < kCols; k += 2)
         pk[k >> 1] = pack_bf16x2(p[k] * (__uint_as_float(r[k]) - dd),
                                  p[k + 1] * (__uint_as_float(r[k + 1]) - dd));
-      tmem_st_32x32b_x32(tDP, pk);
+      tmem_store_part<kCols>(tDP, pk);
       tmem_wait_st();
       tc_fence_before_sync();
       mbar_arrive(ds_ready);
     }
-    // Epilogue: scale * dQ -> bf16; half h writes columns [h*DK/2, (h+1)*DK/2).
-    if (ok && wait_bounded(acc_done, 0, wc)) {
+    // Epilogue: scale * dQ -> bf16; part p < DK/w writes columns [w*p, w*p + w),
+    // w = max(32, DK / parts).
+    constexpr int w = DK / C::kParts > 32 ? DK / C::kParts : 32;
+    if (ok && wait_bounded(acc_done, 0, wc) && part < DK / w) {
       tc_fence_after_sync();
       const bool valid = q0 + row < Nq;
-      __nv_bfloat16* dst = dQ + (size_t(bh) * Nq + size_t(valid ? q0 + row : 0)) * DK + half * (DK / 2);
-      store_row_bf16<DK / 2>(tmem + lanes + C::kTmemDQ + half * (DK / 2), scale, dst, valid);
+      __nv_bfloat16* dst = dQ + (size_t(bh) * Nq + size_t(valid ? q0 + row : 0)) * DK + part * w;
+      store_row_bf16<w>(tmem + lanes + C::kTmemDQ + part * w, scale, dst, valid);
     }
   }
 
@@ -742,7 +780,7 @@ int launch_bwd(const BwdArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
       Dd, int(a.Nq), int(nq_pad), rows_pad);
   cudaError_t e = cudaGetLastError();
   if (e == cudaSuccess) {
-    attn_bwd_dkdv_kernel<DK, DV><<<dim3(unsigned(BH * n_kb)), dim3(kThreads), A::kSmemBytes,
+    attn_bwd_dkdv_kernel<DK, DV><<<dim3(unsigned(BH * n_kb)), dim3(A::kThreads), A::kSmemBytes,
                                    a.stream>>>(
         mq, mk, mv, mdo, nL, Dd, static_cast<__nv_bfloat16*>(a.dK),
         static_cast<__nv_bfloat16*>(a.dV), int(a.Nk), int(nq_pad), int(n_kb), c_log2, a.scale,
@@ -750,7 +788,7 @@ int launch_bwd(const BwdArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
     e = cudaGetLastError();
   }
   if (e == cudaSuccess) {
-    attn_bwd_dq_kernel<DK, DV><<<dim3(unsigned(BH * n_qb)), dim3(kThreads), B::kSmemBytes,
+    attn_bwd_dq_kernel<DK, DV><<<dim3(unsigned(BH * n_qb)), dim3(B::kThreads), B::kSmemBytes,
                                  a.stream>>>(mq, mk, mv, mdo, nL, Dd,
                                              static_cast<__nv_bfloat16*>(a.dQ), int(a.Nq),
                                              int(a.Nk), int(nq_pad), int(n_qb), c_log2, a.scale,
