@@ -120,17 +120,19 @@ int moa_attn_fwd_lse(const void* Q, const void* K, const void* V, void* O, float
  *   LSE      device, float32 [B, H, N_q], the forward pass's log-sum-exp (moa_attn_fwd_lse)
  *   dQ, dK, dV  device, written: [B, H, N_q, d_k], [B, H, N_k, d_k], [B, H, N_k, d_v]
  *   B, H, N_q, N_k, d_k, d_v, scale   as for moa_attn_fwd (the same scale as the forward)
- *   dtype    MOA_BF16 only (MOA_ERR_UNSUPPORTED_DTYPE otherwise); gradients are bf16
+ *   dtype    MOA_BF16 (tensor cores, bf16 gradients) or MOA_FP32 (CUDA cores, fp32
+ *            gradients, no TF32); all eight tensors share it
  *   workspace, workspace_bytes  device scratch of at least moa_attn_bwd_workspace_bytes(...)
  *            bytes, 16-byte aligned, owned by the caller; its contents need no initial value
  *   stream   a cudaStream_t of the current device
- * Supported sizes: d_k, d_v in {64, 128}; the limits of moa_attn_fwd.  Alignment: every
- * tensor 16-byte aligned (LSE 4-byte).  Outputs and workspace must not overlap each other
- * or any input.
+ * Supported sizes: those of moa_attn_fwd for the dtype (bf16: d_k, d_v in {64, 128}; fp32:
+ * d_k, d_v <= 128 and multiples of 4).  Alignment: every tensor 16-byte aligned (LSE 4-byte).
+ * Outputs and workspace must not overlap each other or any input.
  * Behaviour: asynchronous; three kernel launches on `stream` (per-row D and LSE in log2
  * units, then dK/dV, then dQ).  Allocates nothing.  Bounded waits as for moa_attn_fwd
- * (moa_get_device_status reports a timeout).  Accumulation is fp32 in tensor memory; the
- * weights W and dS enter the tensor-core products rounded to bf16.
+ * (moa_get_device_status reports a timeout).  bf16: accumulation is fp32 in tensor memory and
+ * the weights W and dS enter the tensor-core products rounded to bf16.  fp32: every step in
+ * fp32 (expf for the weights).
  */
 int moa_attn_bwd(const void* Q, const void* K, const void* V, const void* O, const void* dO,
                  const float* LSE, void* dQ, void* dK, void* dV, int64_t B, int64_t H,
@@ -139,8 +141,8 @@ int moa_attn_bwd(const void* Q, const void* K, const void* V, const void* O, con
 
 /*
  * moa_attn_bwd_workspace_bytes -- scratch bytes moa_attn_bwd needs: two fp32 values per
- * (b, h) and query row, rows padded to a multiple of 128 (0 for a dtype without a backward
- * or sizes < 1).
+ * (b, h) and query row, rows padded to a multiple of 128, for either dtype (0 for an unknown
+ * dtype or sizes < 1).
  */
 size_t moa_attn_bwd_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int64_t d_k,
                                     int64_t d_v, int dtype);

@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libmoa_attn.so")
 SOURCES = ["moa_attn_api.cu", "attn_fwd_f32_cc.cu", "attn_fwd_bf16_tc.cu", "attn_bwd_bf16_tc.cu",
-           "qkv_proj_bf16_tc.cu"]
+           "attn_bwd_f32_cc.cu", "qkv_proj_bf16_tc.cu"]
 HEADERS = ["internal.h", "ptx.cuh", "tc_common.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xptxas", "-v"]

@@ -132,7 +132,8 @@ __device__ __forceinline__ void store_row_bf16(uint32_t taddr, float mul, __nv_b
 // ------------------------------------------------------------------------------------------
 // Per-row preprocessing
 // ------------------------------------------------------------------------------------------
-// One warp per padded query row r = bh * Nq_pad + i:
+// One group of G = DV/8 lanes per padded query row r = bh * Nq_pad + i (one 16-byte load of O
+// and of dO per lane, 32/G rows per warp):
 //   Dd[r] = sum_c dO[bh,i,c] * O[bh,i,c] (fp32 products of the bf16 values),
 //   nL[r] = -LSE[bh,i] * log2 e;  rows i >= N_q: Dd = 0, nL = -inf.
 template <int DV>
@@ -140,36 +141,35 @@ __global__ void __launch_bounds__(256)
 attn_bwd_pre_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfloat16* __restrict__ dO,
                     const float* __restrict__ lse, float* __restrict__ nL, float* __restrict__ Dd,
                     int Nq, int Nq_pad, long long rows_pad) {
-  const long long r = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+  constexpr int G = DV / 8;      // lanes per row: 8 bf16 (16 bytes) per lane
+  constexpr int kRows = 32 / G;  // rows per warp
   const int lane = threadIdx.x & 31;
-  if (r >= rows_pad) return;
-  const long long bh = r / Nq_pad;
-  const int i = int(r % Nq_pad);
-  if (i >= Nq) {
-    if (lane == 0) {
-      nL[r] = -INFINITY;
-      Dd[r] = 0.f;
-    }
-    return;
-  }
+  const long long r = ((long long)blockIdx.x * 8 + (threadIdx.x >> 5)) * kRows + lane / G;
+  const int gl = lane % G;
+  const bool in_range = r < rows_pad;
+  const long long bh = in_range ? r / Nq_pad : 0;
+  const int i = in_range ? int(r % Nq_pad) : 0;
+  const bool real = in_range && i < Nq;
   const long long src = bh * Nq + i;
   float acc = 0.f;
-  constexpr int kPer = DV / 32;  // bf16 elements per lane: 2 or 4
-  const __nv_bfloat16* o = O + src * DV + lane * kPer;
-  const __nv_bfloat16* g = dO + src * DV + lane * kPer;
+  if (real) {
+    const uint4 ov = *reinterpret_cast<const uint4*>(O + src * DV + gl * 8);
+    const uint4 gv = *reinterpret_cast<const uint4*>(dO + src * DV + gl * 8);
+    const __nv_bfloat162* o2 = reinterpret_cast<const __nv_bfloat162*>(&ov);
+    const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&gv);
 #pragma unroll
-  for (int t = 0; t < kPer; t += 2) {
-    const __nv_bfloat162 ov = *reinterpret_cast<const __nv_bfloat162*>(o + t);
-    const __nv_bfloat162 gv = *reinterpret_cast<const __nv_bfloat162*>(g + t);
-    const float2 of = __bfloat1622float2(ov), gf = __bfloat1622float2(gv);
-    acc = fmaf(of.x, gf.x, acc);
-    acc = fmaf(of.y, gf.y, acc);
+    for (int t = 0; t < 4; ++t) {
+      const float2 of = __bfloat1622float2(o2[t]), gf = __bfloat1622float2(g2[t]);
+      acc = fmaf(of.x, gf.x, acc);
+      acc = fmaf(of.y, gf.y, acc);
+    }
   }
+  // sum over the G lanes of the row (all 32 lanes take part in every shuffle)
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-  if (lane == 0) {
-    nL[r] = -lse[src] * kLog2e;
-    Dd[r] = acc;
+  for (int off = G / 2; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  if (in_range && gl == 0) {
+    nL[r] = real ? -lse[src] * kLog2e : -INFINITY;
+    Dd[r] = real ? acc : 0.f;
   }
 }
 
@@ -775,7 +775,9 @@ int launch_bwd(const BwdArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
   float* Dd = nL + BH * nq_pad;
   const float c_log2 = a.scale * kLog2e;
   const long long rows_pad = BH * nq_pad;
-  attn_bwd_pre_kernel<DV><<<dim3(unsigned((rows_pad + 7) / 8)), dim3(256), 0, a.stream>>>(
+  constexpr int kPreRowsPerBlock = 8 * (32 / (DV / 8));
+  attn_bwd_pre_kernel<DV><<<dim3(unsigned((rows_pad + kPreRowsPerBlock - 1) / kPreRowsPerBlock)),
+                            dim3(256), 0, a.stream>>>(
       static_cast<const __nv_bfloat16*>(a.O), static_cast<const __nv_bfloat16*>(a.dO), a.lse, nL,
       Dd, int(a.Nq), int(nq_pad), rows_pad);
   cudaError_t e = cudaGetLastError();

@@ -85,10 +85,12 @@ struct BwdArgs {
   cudaStream_t stream;
 };
 
-// Workspace of the bf16 backward: per (b,h) and padded query row, D = rowsum(dO * O) and the
-// log-sum-exp in log2 units, fp32.
+// Workspace of the backward: per (b,h) and padded query row, D = rowsum(dO * O) and the
+// log-sum-exp (bf16 path: in log2 units, negated), fp32.
 size_t bwd_workspace_bytes(int64_t B, int64_t H, int64_t Nq);
 int launch_attn_bwd_bf16(const BwdArgs& a, char* msg, size_t msglen);
+// fp32 backward on CUDA cores; same workspace layout (LSE instead of -LSE log2 e in the first half).
+int launch_attn_bwd_f32(const BwdArgs& a, char* msg, size_t msglen);
 // Reads and clears the status word of the backward kernels' bounded waits (after a sync).
 cudaError_t bwd_read_and_clear_status(unsigned* value);
 

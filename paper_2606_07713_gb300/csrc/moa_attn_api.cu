@@ -234,7 +234,7 @@ size_t moa_attn_bwd_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N
   (void)N_k;
   (void)d_k;
   (void)d_v;
-  if (dtype != MOA_BF16 || B <= 0 || H <= 0 || N_q <= 0) return 0;
+  if ((dtype != MOA_BF16 && dtype != MOA_FP32) || B <= 0 || H <= 0 || N_q <= 0) return 0;
   if (moa::numel4(B, H, N_q + 127, 8) < 0) return 0;
   return moa::bwd_workspace_bytes(B, H, N_q);
 }
@@ -248,8 +248,6 @@ int moa_attn_bwd(const void* Q, const void* K, const void* V, const void* O, con
   int64_t sz[4];
   int rc = moa::validate(Q, K, V, const_cast<void*>(O), B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
   if (rc != MOA_OK) return rc;
-  if (dtype != MOA_BF16)
-    return moa::fail(MOA_ERR_UNSUPPORTED_DTYPE, "the backward pass takes bf16 tensors only");
   const void* al[5] = {dO, dQ, dK, dV, workspace};
   for (const void* p : al)
     if (reinterpret_cast<uintptr_t>(p) % 16 != 0)
@@ -277,7 +275,8 @@ int moa_attn_bwd(const void* Q, const void* K, const void* V, const void* O, con
   moa::BwdArgs a{Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v, scale, workspace,
                  static_cast<cudaStream_t>(stream)};
   char msg[256] = {0};
-  rc = moa::launch_attn_bwd_bf16(a, msg, sizeof(msg));
+  rc = dtype == MOA_BF16 ? moa::launch_attn_bwd_bf16(a, msg, sizeof(msg))
+                         : moa::launch_attn_bwd_f32(a, msg, sizeof(msg));
   if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
   moa::t_last_error[0] = '\0';
   return MOA_OK;

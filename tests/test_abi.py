@@ -128,7 +128,8 @@ def test_bwd_workspace_formula(L):
     ws = pkg.moa_attn_bwd_workspace_bytes
     assert ws(2, 3, 200, 300, 64, 64, pkg.MOA_BF16) == 2 * 2 * 3 * 256 * 4
     assert ws(1, 1, 128, 5, 128, 64, pkg.MOA_BF16) == 2 * 128 * 4
-    assert ws(1, 1, 128, 5, 128, 64, pkg.MOA_FP32) == 0
+    assert ws(1, 1, 128, 5, 128, 64, pkg.MOA_FP32) == 2 * 128 * 4      # same layout for fp32
+    assert ws(1, 1, 128, 5, 128, 64, 7) == 0
     assert ws(0, 1, 128, 5, 128, 64, pkg.MOA_BF16) == 0
 
 
@@ -146,8 +147,9 @@ def test_bwd_validation_without_gpu(L):
         q = list(P)
         q[i] = None
         assert call(q) == _lib.MOA_ERR_INVALID_ARG
-    assert call(dtype=0) == _lib.MOA_ERR_UNSUPPORTED_DTYPE
+    assert call(dtype=7) == _lib.MOA_ERR_UNSUPPORTED_DTYPE
     assert call(d=(1, 1, 8, 8, 96, 64, 0.125)) == _lib.MOA_ERR_UNSUPPORTED_SHAPE
+    assert call(dtype=0, d=(1, 1, 8, 8, 132, 64, 0.125)) == _lib.MOA_ERR_UNSUPPORTED_SHAPE
     assert call(ws_bytes=100) == _lib.MOA_ERR_INVALID_ARG               # workspace too small
     q = list(P); q[9] = None
     assert call(q) == _lib.MOA_ERR_INVALID_ARG                          # no workspace
