@@ -13,7 +13,13 @@
 // memory.
 //
 // Layout: Q, K, V, O contiguous row-major [B,H,N,d] float32.
-// CTA: 128 threads = 4 warps, BM = 32 rows (8 per warp), BN = 64 keys.
+// Two kernels:
+//   attn_fwd_f32_cc_kernel   CTA of 128 threads = 4 warps, BM = 32 rows (8 per warp), BN = 64
+//                            keys; K and V tiles shared by the CTA's 32 rows through smem.
+//   attn_fwd_f32_row_kernel  one warp per query row (lane = key of a 32-key chunk for the
+//                            scores, lane = output column for the sum over V), for problems too
+//                            small to give every SM a 32-row CTA: the work spreads over up to
+//                            32x as many warps, which matters when the call is latency-bound.
 #include <cuda_runtime.h>
 #include <math.h>
 #include <cstdio>
@@ -167,9 +173,121 @@ attn_fwd_f32_cc_kernel(const float* __restrict__ Q, const float* __restrict__ K,
   }
 }
 
+// One warp per query row r = (b*H + h)*N_q + i; 8 rows per CTA.
+__global__ void __launch_bounds__(256)
+attn_fwd_f32_row_kernel(const float* __restrict__ Q, const float* __restrict__ K,
+                        const float* __restrict__ V, float* __restrict__ O,
+                        float* __restrict__ lse, int Nq, int Nk, int dk, int dv, float scale,
+                        long long rows) {
+  __shared__ float sq[8][kMaxD];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long r = (long long)blockIdx.x * 8 + warp;
+  if (r >= rows) return;  // whole warps leave together
+  const long long bh = r / Nq;
+  const float* q = Q + r * dk;
+  const float* Kh = K + bh * (long long)Nk * dk;
+  const float* Vh = V + bh * (long long)Nk * dv;
+  for (int j = lane; j < dk; j += 32) sq[warp][j] = q[j];
+  __syncwarp();
+  float m = -INFINITY, l = 0.f;
+  float acc[kMaxColGroups];
+#pragma unroll
+  for (int g = 0; g < kMaxColGroups; ++g) acc[g] = 0.f;
+  for (int k0 = 0; k0 < Nk; k0 += 32) {
+    // lane = key k0 + lane: its score (rows past N_k: -inf)
+    const int key = k0 + lane;
+    float s = -INFINITY;
+    if (key < Nk) {
+      const float* kr = Kh + (long long)key * dk;
+      float d = 0.f;
+      // groups of 4 float4 loads in flight before their products
+      for (int j0 = 0; j0 < dk; j0 += 16) {
+        float4 kv[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          kv[u] = j0 + 4 * u < dk ? *reinterpret_cast<const float4*>(kr + j0 + 4 * u)
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int j = j0 + 4 * u;
+          if (j < dk) {
+            d = fmaf(sq[warp][j], kv[u].x, d);
+            d = fmaf(sq[warp][j + 1], kv[u].y, d);
+            d = fmaf(sq[warp][j + 2], kv[u].z, d);
+            d = fmaf(sq[warp][j + 3], kv[u].w, d);
+          }
+        }
+      }
+      s = d * scale;
+    }
+    float cmax = s;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) cmax = fmaxf(cmax, __shfl_xor_sync(0xffffffffu, cmax, off));
+    const float mnew = fmaxf(m, cmax);       // finite: every chunk has at least one key
+    const float alpha = expf(m - mnew);      // exp(-inf) = 0 on the first chunk
+    const float p = expf(s - mnew);          // 0 for keys past N_k
+    float psum = p;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) psum += __shfl_xor_sync(0xffffffffu, psum, off);
+    l = l * alpha + psum;
+    m = mnew;
+    // lane = output column: acc = alpha * acc + sum over the chunk's keys of p_k V[k, c]
+    const int kn = min(32, Nk - k0);
+#pragma unroll
+    for (int g = 0; g < kMaxColGroups; ++g) acc[g] *= alpha;
+    // eight value rows loaded before their products (keys past N_k read as 0 with p = 0)
+    for (int kb = 0; kb < kn; kb += 8) {
+      float vv[8][kMaxColGroups];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float* vr = Vh + (long long)(k0 + kb + u) * dv;
+#pragma unroll
+        for (int g = 0; g < kMaxColGroups; ++g) {
+          const int c = lane + 32 * g;
+          vv[u][g] = (kb + u < kn && c < dv) ? vr[c] : 0.f;
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float pk = __shfl_sync(0xffffffffu, p, (kb + u) & 31);
+#pragma unroll
+        for (int g = 0; g < kMaxColGroups; ++g) acc[g] = fmaf(pk, vv[u][g], acc[g]);
+      }
+    }
+  }
+  const float inv = 1.0f / l;
+#pragma unroll
+  for (int g = 0; g < kMaxColGroups; ++g) {
+    const int c = lane + 32 * g;
+    if (c < dv) O[r * dv + c] = acc[g] * inv;
+  }
+  if (lse != nullptr && lane == 0) lse[r] = m + logf(l);
+}
+
 }  // namespace
 
 int launch_attn_fwd_f32(const AttnArgs& a, char* msg, size_t msglen) {
+  // Few 32-row CTAs (fewer than two per SM): one warp per row instead.
+  int dev = 0, sms = 148;
+  if (cudaGetDevice(&dev) == cudaSuccess)
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const long long rows = (long long)a.B * a.H * a.Nq;
+  if ((long long)a.B * a.H * ((a.Nq + kBM - 1) / kBM) < 2LL * sms) {
+    if ((rows + 7) / 8 > 0x7fffffffLL) {
+      snprintf(msg, msglen, "fp32 path: too many rows");
+      return 3;
+    }
+    attn_fwd_f32_row_kernel<<<dim3(unsigned((rows + 7) / 8)), dim3(256), 0, a.stream>>>(
+        static_cast<const float*>(a.Q), static_cast<const float*>(a.K),
+        static_cast<const float*>(a.V), static_cast<float*>(a.O), a.lse, int(a.Nq), int(a.Nk),
+        int(a.dk), int(a.dv), a.scale, rows);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) {
+      snprintf(msg, msglen, "fp32 row kernel launch: %s", cudaGetErrorString(e));
+      return 5;
+    }
+    return 0;
+  }
   const int n_qtiles = int((a.Nq + kBM - 1) / kBM);
   const long long grid = (long long)a.B * a.H * n_qtiles;
   if (grid > 0x7fffffffLL) {

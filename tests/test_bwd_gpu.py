@@ -144,3 +144,18 @@ def test_bwd_fp32_parity(oracle, shape):
             continue
         err = rel_err(a, b)
         assert err <= 2e-5, f"{shape} {name}: {err:.3e}"
+
+
+def test_bwd_bench_workload_sampled_heads(oracle):
+    """The backward on bench.py's default workload (bf16 B=4 H=16 N=2048 d=64, the launch
+    configuration `bench.py --pass bwd` times), two whole (b, h) slices checked against the
+    oracle element by element (each slice's gradients depend only on that slice)."""
+    cfg = I.CONFIGS[2]
+    x = I.make_inputs(cfg)
+    g, gb = I.make_grad_output(cfg)
+    dq, dk, dv = run_bwd(x, gb)
+    for (b, h) in [(0, 0), (3, 11)]:
+        ref = oracle.attn_bwd(x.q[b:b + 1, h:h + 1], x.k[b:b + 1, h:h + 1], x.v[b:b + 1, h:h + 1],
+                              g[b:b + 1, h:h + 1], x.scale)
+        got = tuple(t[b:b + 1, h:h + 1] for t in (dq, dk, dv))
+        check_grads(got, ref, f"workload 2 slice ({b},{h})")

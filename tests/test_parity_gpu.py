@@ -98,3 +98,14 @@ def test_bf16_grid_beyond_one_wave(oracle, dk, dv):
     ref, lref = oracle.attn_lse(x.q, x.k, x.v, x.scale)
     assert_close(o.float().cpu().numpy(), ref, "bf16", f"tail d_k={dk} d_v={dv}")
     assert np.max(np.abs(lse.double().cpu().numpy() - lref)) <= 1e-3 * (1 + np.max(np.abs(lref)))
+
+
+def test_fp32_tiled_kernel_on_a_large_grid(oracle):
+    """fp32 problems with at least two 32-row CTAs per SM take the tiled kernel (smaller ones take
+    one warp per row); every row checked."""
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    nq = 32 * ((2 * n_sm + 15) // 16)   # 16 heads x nq/32 CTAs >= 2 per SM
+    cfg = I.custom_config(2, 8, nq, 300, 64, 64, dtype="fp32", seed=41)
+    x = I.make_inputs(cfg)
+    o = run(x)
+    assert_close(o, oracle.attn(x.q, x.k, x.v, x.scale), "fp32", "tiled fp32 kernel")
