@@ -177,11 +177,18 @@ int moa_qkv_proj(const void* X, const void* W, void* Q, void* K, void* V, int64_
  *
  * Defines: as moa_attn_fwd (paper Section 4.1, Eq. attention).  Copies hQ, hK,
  * hV (host memory, ideally page-locked) into the caller's device buffers dQ,
- * dK, dV, runs moa_attn_fwd on them and copies dO back into hO, all enqueued
- * on `stream` in that order.  Sizes, layouts, dtype and alignment rules are
+ * dK, dV, runs the attention on them and copies dO back into hO.  The (b, h)
+ * problems are independent (Remark in Section 4.2), so the call is pipelined
+ * over up to four contiguous ranges of heads: the copies of range c+1 into the
+ * device run on a library-owned side stream while the kernel of range c runs on
+ * `stream`, and each range's output goes back on a second side stream.  Work
+ * already queued on `stream` completes before the first copy starts, and
+ * `stream` completes only after the last copy back, so hO holds the result once
+ * `stream` has been synchronised.  Sizes, layouts, dtype and alignment rules are
  * those of moa_attn_fwd; d* are device pointers owned by the caller, h* host
- * pointers owned by the caller.  Asynchronous: hO holds the result once
- * `stream` has been synchronised.  Allocates nothing.
+ * pointers owned by the caller.  Allocates no memory; the first call on a device
+ * creates the two side streams and their events (kept until the process exits).
+ * Calls on one device enqueue under a lock and share the side streams.
  */
 int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO, void* dQ,
                         void* dK, void* dV, void* dO, int64_t B, int64_t H, int64_t N_q,

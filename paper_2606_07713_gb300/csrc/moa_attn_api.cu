@@ -8,6 +8,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <mutex>
 
 #include "../../include/moa_attn.h"
 #include "internal.h"
@@ -115,6 +116,33 @@ int dispatch(const void* Q, const void* K, const void* V, void* O, int64_t B, in
   return MOA_OK;
 }
 
+// Side streams and events of the pipelined staged call, one set per device, created on the
+// device's first staged call.  The mutex is held while a call enqueues its work, so the events
+// of two concurrent calls never interleave.
+constexpr int kStageChunks = 4;
+constexpr int kMaxDevices = 64;
+struct StagePipe {
+  cudaStream_t copy_in = nullptr, copy_out = nullptr;
+  cudaEvent_t start = nullptr, end = nullptr;
+  cudaEvent_t in_done[kStageChunks] = {}, kern_done[kStageChunks] = {};
+  bool ready = false;
+};
+StagePipe g_pipes[kMaxDevices];
+std::mutex g_pipe_mu[kMaxDevices];
+
+cudaError_t make_pipe(StagePipe& p) {
+  cudaError_t e = cudaStreamCreateWithFlags(&p.copy_in, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p.copy_out, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p.start, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p.end, cudaEventDisableTiming);
+  for (int c = 0; e == cudaSuccess && c < kStageChunks; ++c) {
+    e = cudaEventCreateWithFlags(&p.in_done[c], cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p.kern_done[c], cudaEventDisableTiming);
+  }
+  p.ready = e == cudaSuccess;
+  return e;
+}
+
 }  // namespace
 }  // namespace moa
 
@@ -155,18 +183,66 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
   int rc = moa::validate(dQ, dK, dV, dO, B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
   if (rc != MOA_OK) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= moa::kMaxDevices)
+    return moa::fail(MOA_ERR_CUDA, "no usable current device: %s", cudaGetErrorString(e));
+  // The (b, h) problems are independent, so the call is pipelined over head ranges: the
+  // host-to-device copies of range c+1 (side stream) overlap the kernel of range c (`stream`),
+  // whose output goes back on a second side stream while later ranges compute.
+  std::lock_guard<std::mutex> lock(moa::g_pipe_mu[dev]);
+  moa::StagePipe& p = moa::g_pipes[dev];
+  if (!p.ready && (e = moa::make_pipe(p)) != cudaSuccess)
+    return moa::fail(MOA_ERR_CUDA, "staged pipeline set-up: %s", cudaGetErrorString(e));
+  const int64_t BH = B * H;
+  const int chunks = int(BH < moa::kStageChunks ? BH : moa::kStageChunks);
+  const int64_t per = (BH + chunks - 1) / chunks;
+  const int64_t elt = dtype == MOA_FP32 ? 4 : 2;
+  const int64_t row_bytes[4] = {N_q * d_k * elt, N_k * d_k * elt, N_k * d_v * elt, N_q * d_v * elt};
   const void* src[3] = {hQ, hK, hV};
   void* dst[3] = {dQ, dK, dV};
-  for (int i = 0; i < 3; ++i) {
-    cudaError_t e = cudaMemcpyAsync(dst[i], src[i], size_t(sz[i]), cudaMemcpyHostToDevice, s);
-    if (e != cudaSuccess)
-      return moa::fail(MOA_ERR_CUDA, "host-to-device copy: %s", cudaGetErrorString(e));
+  auto chk = [&](cudaError_t err, const char* what) {
+    if (err != cudaSuccess) moa::fail(MOA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(err));
+    return err == cudaSuccess;
+  };
+  // Work already queued on `stream` (e.g. a kernel still reading dQ) finishes before the copies.
+  if (!chk(cudaEventRecord(p.start, s), "event record") ||
+      !chk(cudaStreamWaitEvent(p.copy_in, p.start, 0), "stream wait"))
+    return MOA_ERR_CUDA;
+  for (int c = 0; c < chunks; ++c) {
+    const int64_t h0 = c * per, nh = (h0 + per <= BH ? per : BH - h0);
+    if (nh <= 0) break;
+    for (int t = 0; t < 3; ++t)
+      if (!chk(cudaMemcpyAsync(static_cast<char*>(dst[t]) + h0 * row_bytes[t],
+                               static_cast<const char*>(src[t]) + h0 * row_bytes[t],
+                               size_t(nh * row_bytes[t]), cudaMemcpyHostToDevice, p.copy_in),
+               "host-to-device copy"))
+        return MOA_ERR_CUDA;
+    if (!chk(cudaEventRecord(p.in_done[c], p.copy_in), "event record")) return MOA_ERR_CUDA;
   }
-  rc = moa::dispatch(dQ, dK, dV, dO, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream);
-  if (rc != MOA_OK) return rc;
-  cudaError_t e = cudaMemcpyAsync(hO, dO, size_t(sz[3]), cudaMemcpyDeviceToHost, s);
-  if (e != cudaSuccess)
-    return moa::fail(MOA_ERR_CUDA, "device-to-host copy: %s", cudaGetErrorString(e));
+  for (int c = 0; c < chunks; ++c) {
+    const int64_t h0 = c * per, nh = (h0 + per <= BH ? per : BH - h0);
+    if (nh <= 0) break;
+    if (!chk(cudaStreamWaitEvent(s, p.in_done[c], 0), "stream wait")) return MOA_ERR_CUDA;
+    rc = moa::dispatch(static_cast<const char*>(dQ) + h0 * row_bytes[0],
+                       static_cast<const char*>(dK) + h0 * row_bytes[1],
+                       static_cast<const char*>(dV) + h0 * row_bytes[2],
+                       static_cast<char*>(dO) + h0 * row_bytes[3], 1, nh, N_q, N_k, d_k, d_v,
+                       scale, dtype, stream);
+    if (rc != MOA_OK) return rc;
+    if (!chk(cudaEventRecord(p.kern_done[c], s), "event record") ||
+        !chk(cudaStreamWaitEvent(p.copy_out, p.kern_done[c], 0), "stream wait") ||
+        !chk(cudaMemcpyAsync(static_cast<char*>(hO) + h0 * row_bytes[3],
+                             static_cast<const char*>(dO) + h0 * row_bytes[3],
+                             size_t(nh * row_bytes[3]), cudaMemcpyDeviceToHost, p.copy_out),
+             "device-to-host copy"))
+      return MOA_ERR_CUDA;
+  }
+  // `stream` completes only after the last copy back: synchronising it makes hO valid.
+  if (!chk(cudaEventRecord(p.end, p.copy_out), "event record") ||
+      !chk(cudaStreamWaitEvent(s, p.end, 0), "stream wait"))
+    return MOA_ERR_CUDA;
+  moa::t_last_error[0] = '\0';
   return MOA_OK;
 }
 

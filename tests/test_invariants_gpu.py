@@ -132,3 +132,28 @@ def test_errors_reported_through_binding():
     with pytest.raises(pkg.MoaError) as e:
         pkg.attn_fwd(q96, q96, v)
     assert e.value.status == 3
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_staged_pipeline_back_to_back_on_one_stream(dtype):
+    """Two staged calls back to back on one user stream, sharing the device buffers: the second
+    call's copies must wait for the first call's kernels, and synchronising that stream alone
+    must make both host outputs valid.  9 heads: ranges of 3, 3, 3 (one range empty)."""
+    shape = (3, 3, 200, 300, 64, 64)
+    x1 = I.make_inputs(I.custom_config(*shape, dtype=dtype, seed=51))
+    x2 = I.make_inputs(I.custom_config(*shape, dtype=dtype, seed=52))
+    ref1 = pkg.attn_fwd(*to_device(x1)).cpu()
+    ref2 = pkg.attn_fwd(*to_device(x2)).cpu()
+    torch.cuda.synchronize()
+    h1 = [t.cpu().pin_memory() for t in to_device(x1)]
+    h2 = [t.cpu().pin_memory() for t in to_device(x2)]
+    dq, dk, dv = (torch.empty_like(t) for t in to_device(x1))
+    do = torch.empty(ref1.shape, dtype=ref1.dtype, device="cuda")
+    ho1 = torch.empty(ref1.shape, dtype=ref1.dtype).pin_memory()
+    ho2 = torch.empty(ref1.shape, dtype=ref1.dtype).pin_memory()
+    s = torch.cuda.Stream()
+    pkg.attn_fwd_staged(*h1, ho1, dq, dk, dv, do, stream=s)
+    pkg.attn_fwd_staged(*h2, ho2, dq, dk, dv, do, stream=s)
+    s.synchronize()
+    assert torch.equal(ho1, ref1)
+    assert torch.equal(ho2, ref2)
