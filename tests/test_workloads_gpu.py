@@ -48,7 +48,15 @@ def test_workload(oracle, cid):
         rows = sample_rows(x)
         ref = oracle.rows(x.q, x.k, x.v, x.scale, rows)
         got = o.float().reshape(-1, s.d_v)[torch.from_numpy(rows).to(o.device)].cpu().numpy()
-    assert_close(got, ref, x.cfg.dtype, f"workload {cid}")
+    err = assert_close(got, ref, x.cfg.dtype, f"workload {cid}")
+    # also the relative RMS error and the worst row (reported; the bound above is the test)
+    d = got.astype(np.float64) - ref
+    rms = float(np.sqrt(np.mean(d * d)) / np.sqrt(np.mean(ref * ref)))
+    worst = int(np.argmax(np.max(np.abs(d), axis=1)))
+    wrow = worst if full else int(rows[worst])
+    b, rem = divmod(wrow, s.H * s.N_q)
+    h, i = divmod(rem, s.N_q)
+    print(f"workload {cid}: max rel err {err:.2e}, rel RMS {rms:.2e}, worst row (b={b}, h={h}, i={i})")
     if x.plants:
         # One dominant key (margin > 30 in the scores): the output row is that key's value row.
         sc = oracle.scores(x.q[0, 0, [p[2] for p in x.plants if p[1] == 0]], x.k[0, 0], x.scale)
