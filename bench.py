@@ -299,8 +299,14 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
             "clocks": clocks,
             "wall_s_timed_loop": round(wall, 4),
         }
+        line["ms_median"] = round(float(np.median(kern_ms)), 6)
+        line["ms_best"] = round(float(np.min(kern_ms)), 6)
+        if cfg.dtype == "bf16":
+            sus = float(peaks.get("bf16_tflops_sustained", 1700.0))
+            line["pct_of_bf16_peak_sustained"] = round(100.0 * achieved / sus, 2)
         if world == 1:
-            line["cpu_baseline"] = cpu_baseline(cfg, x, budget_s=args.cpu_budget)
+            line["cpu_baseline"] = cpu_baseline(cfg, x, budget_s=args.cpu_budget,
+                                                gpu_out=o.float().reshape(-1, s.d_v))
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
@@ -690,7 +696,9 @@ def _cores() -> int:
         return os.cpu_count() or 1
 
 
-def cpu_baseline(cfg, x, budget_s: float = 12.0) -> dict:
+def cpu_baseline(cfg, x, budget_s: float = 12.0, gpu_out=None) -> dict:
+    """The oracle timed on the host cores over a seeded row sample.  If the GPU output (rows of
+    [B*H*N_q, d_v]) is given, the same sampled rows also give the run's parity error."""
     import oracle
     orc = oracle.get()
     s = cfg.shape
@@ -703,11 +711,18 @@ def cpu_baseline(cfg, x, budget_s: float = 12.0) -> dict:
     n = int(min(total, max(256, len(probe) * budget_s / max(dt, 1e-6))))
     rows = _oracle_rows(cfg, x, n, 2)
     t0 = time.perf_counter()
-    orc.rows(x.q, x.k, x.v, cfg.scale, rows)
+    ref = orc.rows(x.q, x.k, x.v, cfg.scale, rows)
     dt = time.perf_counter() - t0
-    return {"value": round(flops_row * len(rows) / dt / 1e12, 6), "unit": "TFLOP/s",
-            "cores": orc.max_threads(), "kind": "oracle",
-            "sample": f"{len(rows)} of {total} output rows (seeded, uniform), fp64, {dt:.1f} s"}
+    out = {"value": round(flops_row * len(rows) / dt / 1e12, 6), "unit": "TFLOP/s",
+           "cores": orc.max_threads(), "kind": "oracle",
+           "sample": f"{len(rows)} of {total} output rows (seeded, uniform), fp64, {dt:.1f} s"}
+    if gpu_out is not None:
+        import torch
+        got = gpu_out[torch.from_numpy(rows).to(gpu_out.device)].cpu().numpy().astype(np.float64)
+        d = got - ref
+        out["sampled_max_rel_err"] = float(np.max(np.abs(d)) / np.max(np.abs(ref)))
+        out["sampled_rel_rms_err"] = float(np.sqrt(np.mean(d * d)) / np.sqrt(np.mean(ref * ref)))
+    return out
 
 
 def run_reference(args, cfg: I.AttnConfig) -> None:

@@ -9,6 +9,12 @@
  *
  * Shared library: libmoa_attn.so (plain C ABI, no C++ or PyTorch types).
  * Every entry point is thread-safe; moa_last_error() is per calling thread.
+ *
+ * Environment (read once per process):
+ *   MOA_WAIT_LIMIT_NS  limit of one bounded wait inside a kernel (default 1e9 ns)
+ *   MOA_DEBUG_SYNC=1   every entry point synchronises its stream after launching and returns
+ *                      MOA_ERR_CUDA or MOA_ERR_DEVICE_TIMEOUT for that call itself (debugging;
+ *                      off by default, when errors surface at moa_get_device_status)
  */
 #ifndef MOA_ATTN_H
 #define MOA_ATTN_H

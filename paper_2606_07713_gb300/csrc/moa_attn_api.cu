@@ -104,6 +104,30 @@ int validate(const void* Q, const void* K, const void* V, void* O, int64_t B, in
   return MOA_OK;
 }
 
+// MOA_DEBUG_SYNC=1: every entry point synchronises its stream after launching and reports a
+// CUDA error or a recorded wait timeout from that call directly (debugging aid; off by default).
+bool debug_sync() {
+  static const bool v = [] {
+    const char* s = std::getenv("MOA_DEBUG_SYNC");
+    return s && *s && std::strcmp(s, "0") != 0;
+  }();
+  return v;
+}
+
+int debug_check(void* stream) {
+  if (!debug_sync()) return MOA_OK;
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return fail(MOA_ERR_CUDA, "debug sync: %s", cudaGetErrorString(e));
+  unsigned v = 0, vb = 0, vp = 0;
+  e = bf16_read_and_clear_status(&v);
+  if (e == cudaSuccess) e = bwd_read_and_clear_status(&vb);
+  if (e == cudaSuccess) e = proj_read_and_clear_status(&vp);
+  if (e != cudaSuccess) return fail(MOA_ERR_CUDA, "debug status read: %s", cudaGetErrorString(e));
+  if ((v | vb | vp) != 0)
+    return fail(MOA_ERR_DEVICE_TIMEOUT, "debug sync: a kernel wait ran out (status %u)", v | vb | vp);
+  return MOA_OK;
+}
+
 int dispatch(const void* Q, const void* K, const void* V, void* O, int64_t B, int64_t H,
              int64_t Nq, int64_t Nk, int64_t dk, int64_t dv, float scale, int dtype,
              void* stream, float* lse = nullptr) {
@@ -113,7 +137,7 @@ int dispatch(const void* Q, const void* K, const void* V, void* O, int64_t B, in
                                    : launch_attn_fwd_f32(a, msg, sizeof(msg));
   if (rc != MOA_OK) return fail(rc, "%s", msg);
   t_last_error[0] = '\0';
-  return MOA_OK;
+  return debug_check(stream);
 }
 
 // Side streams and events of the pipelined staged call, one set per device, created on the
@@ -284,7 +308,7 @@ int moa_attn_fwd_splitkv(const void* Q, const void* K, const void* V, void* O, i
   rc = moa::launch_attn_fwd_bf16_split(a, sp, workspace, msg, sizeof(msg));
   if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
   moa::t_last_error[0] = '\0';
-  return MOA_OK;
+  return moa::debug_check(stream);
 }
 
 int moa_attn_fwd_splitkv_noalloc(const void* Q, const void* K, const void* V, void* O, int64_t B,
@@ -302,7 +326,7 @@ int moa_attn_fwd_splitkv_noalloc(const void* Q, const void* K, const void* V, vo
                                                sizeof(msg));
   if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
   moa::t_last_error[0] = '\0';
-  return MOA_OK;
+  return moa::debug_check(stream);
 }
 
 size_t moa_attn_bwd_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int64_t d_k,
@@ -355,7 +379,7 @@ int moa_attn_bwd(const void* Q, const void* K, const void* V, const void* O, con
                          : moa::launch_attn_bwd_f32(a, msg, sizeof(msg));
   if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
   moa::t_last_error[0] = '\0';
-  return MOA_OK;
+  return moa::debug_check(stream);
 }
 
 int moa_qkv_proj(const void* X, const void* W, void* Q, void* K, void* V, int64_t B, int64_t N,
@@ -397,7 +421,7 @@ int moa_qkv_proj(const void* X, const void* W, void* Q, void* K, void* V, int64_
   const int rc = moa::launch_qkv_proj_bf16(a, msg, sizeof(msg));
   if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
   moa::t_last_error[0] = '\0';
-  return MOA_OK;
+  return moa::debug_check(stream);
 }
 
 const char* moa_last_error(void) { return moa::t_last_error; }
