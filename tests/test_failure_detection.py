@@ -41,6 +41,9 @@ def test_debug_sync_mode_runs_every_entry_point_synchronously():
     import os
     import subprocess
     import sys
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
     code = (
         "import torch, paper_2606_07713_gb300 as p\n"
         "q = torch.randn(1, 2, 300, 64, device='cuda', dtype=torch.bfloat16)\n"
