@@ -213,16 +213,28 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
  * few 256-row query blocks to fill the GPU (long keys, short queries).
  *
  * Arguments: as moa_attn_fwd, plus
- *   num_splits       requested number of key ranges (>= 1; fewer are used when N_k has fewer
- *                    128-key blocks; 1 runs the unsplit kernel)
+ *   num_splits       requested number of key ranges for every 256-row query block (>= 1;
+ *                    fewer are used when N_k has fewer 128-key blocks; 1 runs the unsplit
+ *                    kernel), or MOA_SPLITS_AUTO (see below)
  *   workspace        device pointer, 16-byte aligned, not overlapping any tensor; owned by the
  *                    caller; contents on entry are ignored and undefined afterwards
- *   workspace_bytes  its size; must be >= moa_attn_splitkv_workspace_bytes(...)
+ *   workspace_bytes  its size; must be >= moa_attn_splitkv_workspace_bytes(...) with the same
+ *                    num_splits (and, for MOA_SPLITS_AUTO, the same current device)
+ * MOA_SPLITS_AUTO: the library chooses from the current device's SM count.  When the
+ * B*H*ceil(N_q/256) query blocks (one CTA per SM each) leave SMs idle, every block's key axis
+ * is split so that the CTAs fill the SMs (at least two key blocks per range), when a model of
+ * the split's cost predicts a saving of at least 15 %; with a full wave of blocks or more
+ * nothing is split and the call is moa_attn_fwd (same bits).  moa_attn_split_plan reports
+ * the choice.
  * MOA_FP32 has no split form: the call then computes the same result with moa_attn_fwd.
- * Errors: those of moa_attn_fwd; MOA_ERR_INVALID_ARG for num_splits < 1 or a missing, too
- * small or overlapping workspace; MOA_ERR_MISALIGNED for a misaligned workspace.
- * Asynchronous on `stream`; allocates nothing.
+ * Errors: those of moa_attn_fwd; MOA_ERR_INVALID_ARG for num_splits < 0 or a missing, too
+ * small or overlapping workspace; MOA_ERR_MISALIGNED for a misaligned workspace;
+ * MOA_ERR_CUDA when MOA_SPLITS_AUTO cannot read the current device's SM count.
+ * Asynchronous on `stream`; allocates nothing.  Launches the split kernel and the merge, or
+ * the unsplit kernel alone.
  */
+#define MOA_SPLITS_AUTO 0
+
 int moa_attn_fwd_splitkv(const void* Q, const void* K, const void* V, void* O, int64_t B,
                          int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v,
                          float scale, int dtype, int num_splits, void* workspace,
@@ -230,12 +242,27 @@ int moa_attn_fwd_splitkv(const void* Q, const void* K, const void* V, void* O, i
 
 /*
  * moa_attn_splitkv_workspace_bytes -- bytes of workspace moa_attn_fwd_splitkv needs for these
- * sizes and this requested split count: splits * B*H*N_q * (4*d_v + 8) (fp32 partial rows plus
- * a running maximum and sum per row and split), 0 when no split happens or for MOA_FP32 or
- * invalid sizes.
+ * sizes and this num_splits: splits * B*H*N_q * (4*d_v + 8) (fp32 partial rows plus a
+ * running maximum and sum per row and split).  0 when no split happens, for MOA_FP32, for
+ * invalid sizes, and for MOA_SPLITS_AUTO without a usable current device.
  */
 size_t moa_attn_splitkv_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k,
                                         int64_t d_k, int64_t d_v, int dtype, int num_splits);
+
+/*
+ * moa_attn_split_plan -- the schedule moa_attn_fwd_splitkv would run (host only).
+ *
+ * For these sizes and num_splits (>= 1, or MOA_SPLITS_AUTO) on a GPU of sm_count SMs
+ * (<= 0: the current device, which then must be usable), writes through each non-null
+ * pointer: *splits, the key ranges per split query block (1: nothing is split);
+ * *key_blocks_per_split, the 128-key blocks in each range (the last may hold fewer); and
+ * *whole_query_blocks, how many 256-row query blocks run unsplit (all or none of them).
+ * Launches nothing.  Errors: MOA_ERR_INVALID_ARG for non-positive or overflowing sizes or
+ * num_splits < 0; MOA_ERR_CUDA when sm_count <= 0 and no device answers.
+ */
+int moa_attn_split_plan(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int num_splits,
+                        int sm_count, int* splits, int* key_blocks_per_split,
+                        int64_t* whole_query_blocks);
 
 /* Size in bytes of the fixed device array used by moa_attn_fwd_splitkv_noalloc (16 MiB). */
 #define MOA_NOALLOC_SCRATCH_BYTES ((size_t)16 << 20)
@@ -256,7 +283,8 @@ size_t moa_attn_splitkv_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64
  * Result and arguments: exactly those of moa_attn_fwd_splitkv without the workspace; the
  * caller still passes Q, K, V and O.  A split whose partials need more than
  * MOA_NOALLOC_SCRATCH_BYTES (splits * B*H*N_q * (4*d_v + 8) bytes) is rejected with
- * MOA_ERR_UNSUPPORTED_SHAPE and a message naming both sizes; nothing is launched.
+ * MOA_ERR_UNSUPPORTED_SHAPE and a message naming both sizes; nothing is launched.  With
+ * MOA_SPLITS_AUTO a plan that would not fit runs unsplit instead.
  *
  * The first call on a device looks up that device's address of the array (once per device,
  * with the device current); make that first call before any stream capture on the device.

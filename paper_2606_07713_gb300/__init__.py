@@ -17,7 +17,8 @@ from ._lib import (MOA_BF16, MOA_FP32, MoaError, check, lib, moa_attn_dnf_bytes,
                    moa_attn_flops, moa_attn_fwd, moa_attn_fwd_staged, moa_attn_version,
                    moa_get_device_status, moa_last_error, moa_selftest_wait_timeout,
                    moa_attn_fwd_splitkv, moa_attn_splitkv_workspace_bytes, moa_attn_fwd_lse,
-                   moa_attn_bwd, moa_attn_bwd_workspace_bytes, moa_qkv_proj)
+                   moa_attn_bwd, moa_attn_bwd_workspace_bytes, moa_qkv_proj,
+                   moa_attn_split_plan, MOA_SPLITS_AUTO)
 
 __all__ = ["attn_fwd", "attn_fwd_staged", "get_device_status", "attn_flops", "dnf_bytes",
            "MOA_FP32", "MOA_BF16", "MoaError", "moa_attn_fwd", "moa_attn_fwd_staged",
@@ -25,7 +26,7 @@ __all__ = ["attn_fwd", "attn_fwd_staged", "get_device_status", "attn_flops", "dn
            "moa_attn_version", "moa_selftest_wait_timeout", "attn_fwd_splitkv",
            "moa_attn_fwd_splitkv", "moa_attn_splitkv_workspace_bytes", "attn_fwd_lse",
            "moa_attn_fwd_lse", "attn_bwd", "moa_attn_bwd", "moa_attn_bwd_workspace_bytes",
-           "qkv_proj", "moa_qkv_proj"]
+           "qkv_proj", "moa_qkv_proj", "moa_attn_split_plan", "MOA_SPLITS_AUTO"]
 
 
 def _dtype_code(t) -> int:
@@ -165,11 +166,12 @@ def qkv_proj(x, w, H: int, d_k: int, d_v: int, out=None, stream=None):
     return q, k, v
 
 
-def attn_fwd_splitkv(q, k, v, num_splits: int, scale: float | None = None, out=None,
-                     workspace=None, stream=None):
-    """attn_fwd with the key axis split into up to num_splits ranges merged at the end.  The
-    workspace (a CUDA uint8 tensor of at least moa_attn_splitkv_workspace_bytes(...) bytes) is
-    allocated here when not given."""
+def attn_fwd_splitkv(q, k, v, num_splits: int = MOA_SPLITS_AUTO, scale: float | None = None,
+                     out=None, workspace=None, stream=None):
+    """attn_fwd with the key axis split into up to num_splits ranges merged at the end; with
+    MOA_SPLITS_AUTO (0) only the query blocks of the last partial wave are split, as the library
+    chooses for q's device.  The workspace (a CUDA uint8 tensor of at least
+    moa_attn_splitkv_workspace_bytes(...) bytes) is allocated here when not given."""
     import torch
     for t in (q, k, v):
         if not t.is_cuda or not t.is_contiguous():
@@ -182,10 +184,10 @@ def attn_fwd_splitkv(q, k, v, num_splits: int, scale: float | None = None, out=N
         scale = 1.0 / math.sqrt(dk)
     if out is None:
         out = torch.empty((B, H, Nq, dv), dtype=q.dtype, device=q.device)
-    need = moa_attn_splitkv_workspace_bytes(B, H, Nq, Nk, dk, dv, code, int(num_splits))
-    if workspace is None:
-        workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=q.device)
     with torch.cuda.device(q.device):
+        need = moa_attn_splitkv_workspace_bytes(B, H, Nq, Nk, dk, dv, code, int(num_splits))
+        if workspace is None:
+            workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=q.device)
         s = stream if stream is not None else torch.cuda.current_stream(q.device)
         check(moa_attn_fwd_splitkv(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), B, H,
                                    Nq, Nk, dk, dv, float(scale), code, int(num_splits),

@@ -57,6 +57,10 @@ SIGNATURES = {
     "moa_attn_fwd_splitkv_noalloc": (ctypes.c_int, [_VP, _VP, _VP, _VP, _I64, _I64, _I64, _I64,
                                                     _I64, _I64, ctypes.c_float, ctypes.c_int,
                                                     ctypes.c_int, _VP]),
+    "moa_attn_split_plan": (ctypes.c_int, [_I64, _I64, _I64, _I64, ctypes.c_int, ctypes.c_int,
+                                           ctypes.POINTER(ctypes.c_int),
+                                           ctypes.POINTER(ctypes.c_int),
+                                           ctypes.POINTER(ctypes.c_int64)]),
     "moa_last_error": (ctypes.c_char_p, []),
     "moa_get_device_status": (ctypes.c_int, [_VP]),
     "moa_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_uint64, _VP]),
@@ -148,8 +152,18 @@ def moa_attn_fwd_splitkv_noalloc(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dt
                                               num_splits, stream)
 
 
-# MOA_NOALLOC_SCRATCH_BYTES of include/moa_attn.h
+def moa_attn_split_plan(B, H, N_q, N_k, num_splits, sm_count) -> tuple[int, int, int, int]:
+    """(status, splits, key_blocks_per_split, whole_query_blocks) of moa_attn_split_plan."""
+    s, per = ctypes.c_int(0), ctypes.c_int(0)
+    whole = ctypes.c_int64(0)
+    rc = lib().moa_attn_split_plan(B, H, N_q, N_k, num_splits, sm_count, ctypes.byref(s),
+                                   ctypes.byref(per), ctypes.byref(whole))
+    return rc, s.value, per.value, whole.value
+
+
+# MOA_NOALLOC_SCRATCH_BYTES and MOA_SPLITS_AUTO of include/moa_attn.h
 MOA_NOALLOC_SCRATCH_BYTES = 16 << 20
+MOA_SPLITS_AUTO = 0
 
 
 def moa_last_error() -> str:

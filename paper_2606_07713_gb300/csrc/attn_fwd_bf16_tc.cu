@@ -167,6 +167,11 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   auto p_free = [&](int j) { return bar0 + 8u * (2 * C::kStages + 9 + j); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
+  // Split instance only: keys from this CTA's first key block to the end of the key axis, and
+  // its key range.  Read from shared memory where needed, so that no register holds them
+  // across the key loop (held in registers they made the split instance spill).
+  volatile int* keys_from = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 8);
+  volatile int* split_s = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 12);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -195,6 +200,10 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(p_free(j), 1);
     }
     *abort_flag = 0;
+    if constexpr (SPLIT) {
+      *keys_from = Nk - kb0 * kBN;
+      *split_s = split;
+    }
     fence_barrier_init();
   }
   if (warp == kMmaWarp0) {
@@ -470,7 +479,8 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         mbar_arrive(s_free(j));
       }
       float* s = reinterpret_cast<float*>(sr);
-      const int valid = min(kBN, Nk - (kb0 + n) * kBN);
+      // Keys of this tile that exist.
+      const int valid = SPLIT ? min(kBN, *keys_from - n * kBN) : min(kBN, Nk - (kb0 + n) * kBN);
       // Step I: maximum of the scaled scores of this tile (max of s if c >= 0, else of -s).
       float tmax;
       if (valid == kBN) {
@@ -553,18 +563,18 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     if (SPLIT && ok && wait_bounded(o_done(j), 0, wc)) {
       tc_fence_after_sync();
       const int grow = q0 + j * kBM + row;
-      const size_t prow = (size_t(split) * (gridDim.x / n_splits / n_qblocks) + bh) * Nq + grow;
+      const size_t prow = (size_t(*split_s) * (gridDim.x / n_splits / n_qblocks) + bh) * Nq + grow;
       float* orow = ws_o + prow * DV;
 #pragma unroll
-      for (int c = 0; c < DV; c += 32) {
-        uint32_t o[32];
-        tmem_ld_32x32b_x32(tO + c, o);
+      for (int c = 0; c < DV; c += 16) {
+        uint32_t o[16];
+        tmem_ld_32x32b_x16(tO + c, o);
         tmem_wait_ld();
-        reg_anchor_x32(o);
+        reg_anchor_x16(o);
         if (grow < Nq) {
           float4* dst = reinterpret_cast<float4*>(orow + c);
 #pragma unroll
-          for (int i = 0; i < 8; ++i)
+          for (int i = 0; i < 4; ++i)
             dst[i] = make_float4(__uint_as_float(o[4 * i]), __uint_as_float(o[4 * i + 1]),
                                  __uint_as_float(o[4 * i + 2]), __uint_as_float(o[4 * i + 3]));
         }
@@ -782,6 +792,36 @@ SplitPlan plan_splits(int64_t Nk, int requested) {
   sp.kv_per_split = int(per);
   sp.n_splits = int((n_kt + per - 1) / per);  // every split gets at least one key block
   return sp;
+}
+
+static_assert(kQTiles * kBM == kQBlockRows, "query block size");
+
+// Model: a whole query block takes time 1; a split of `per` of its n_kt key blocks takes
+// per/n_kt + kSplitFixed (the Q load, the pipeline fill and drain, and the fp32 partial rows,
+// measured at about 0.08 of a 16-block CTA).  The split CTAs of t blocks run as
+// ceil(t * splits / sms) rounds.  Splitting only pays when the blocks leave SMs idle: with a
+// full wave or more, every split CTA adds its fixed cost and the merge to work that already
+// fills the GPU (measured slower on every such shape tried).  Splits keep >= 2 key blocks.
+SplitPlan plan_splits_auto(int64_t units, int64_t Nk, int sms) {
+  constexpr double kSplitFixed = 0.08;
+  constexpr int kMaxSplits = 32;
+  SplitPlan none;
+  if (units <= 0 || Nk <= 0 || sms <= 0 || units >= sms) return none;
+  const int64_t n_kt = (Nk + kBN - 1) / kBN;
+  double best = 1.0;  // one round of whole blocks
+  SplitPlan pick = none;
+  for (int64_t s = 2; s <= kMaxSplits && s <= n_kt / 2; ++s) {
+    const int64_t per = (n_kt + s - 1) / s;
+    const int64_t used = (n_kt + per - 1) / per;
+    const double rounds = double((units * used + sms - 1) / sms);
+    const double est = rounds * (double(per) / double(n_kt) + kSplitFixed);
+    if (est < best - 0.02) {
+      best = est;
+      pick.n_splits = int(used);
+      pick.kv_per_split = int(per);
+    }
+  }
+  return best <= 0.85 ? pick : none;
 }
 
 size_t splitkv_workspace_bytes(int64_t rows, int64_t dv, const SplitPlan& sp) {

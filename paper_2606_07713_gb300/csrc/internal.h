@@ -20,6 +20,9 @@ struct AttnArgs {
   float* lse = nullptr;
 };
 
+// Query rows per CTA of the bf16 forward (one "query block", the unit of its grid).
+constexpr int64_t kQBlockRows = 256;
+
 // How the key axis of the bf16 kernel is split: n_splits contiguous ranges of kv_per_split
 // 128-key blocks (the last may be shorter); n_splits == 1 means no split.
 struct SplitPlan {
@@ -30,8 +33,16 @@ struct SplitPlan {
 // At most `requested` splits, each of at least one key block.
 SplitPlan plan_splits(int64_t Nk, int requested);
 
+// The library's own choice for `units` query blocks on `sms` SMs (one CTA per SM): when the
+// blocks fill less than one wave, every block's key axis is split so that the CTAs fill the
+// SMs; otherwise no split (see the model in the definition).
+SplitPlan plan_splits_auto(int64_t units, int64_t Nk, int sms);
+
 // Workspace of a split bf16 call: fp32 partial rows and (m, l) per split and output row.
 size_t splitkv_workspace_bytes(int64_t rows, int64_t dv, const SplitPlan& sp);
+
+// SM count of the current device, asked once per device.
+cudaError_t device_sm_count(int* sms);
 
 // Size of the fixed device array behind the allocation-free split entry point (16 MiB).
 constexpr size_t kNoallocScratchBytes = size_t(16) << 20;

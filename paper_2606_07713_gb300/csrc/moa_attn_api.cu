@@ -28,6 +28,28 @@ uint64_t wait_limit_ns() {
 }
 
 namespace {
+std::mutex g_sm_mu;
+int g_sm_count[64] = {};
+}  // namespace
+
+cudaError_t device_sm_count(int* sms) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_sm_mu);
+  if (g_sm_count[dev] <= 0) {
+    int n = 0;
+    e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    if (n <= 0) return cudaErrorInvalidDevice;
+    g_sm_count[dev] = n;
+  }
+  *sms = g_sm_count[dev];
+  return cudaSuccess;
+}
+
+namespace {
 
 thread_local char t_last_error[512] = {0};
 
@@ -167,6 +189,32 @@ cudaError_t make_pipe(StagePipe& p) {
   return e;
 }
 
+int current_sm_count(int* sms) {
+  const cudaError_t e = device_sm_count(sms);
+  if (e != cudaSuccess)
+    return fail(MOA_ERR_CUDA, "SM count of the current device: %s", cudaGetErrorString(e));
+  return MOA_OK;
+}
+
+// The split of a bf16 call: num_splits splits of every query block, or for MOA_SPLITS_AUTO the
+// library's choice for `sms` SMs (sms <= 0: the current device's count).
+int choose_plan(int64_t B, int64_t H, int64_t Nq, int64_t Nk, int num_splits, int sms,
+                SplitPlan* sp) {
+  if (num_splits < 0) return fail(MOA_ERR_INVALID_ARG, "num_splits must be >= 0");
+  if (num_splits > 0) {
+    *sp = plan_splits(Nk, num_splits);
+    return MOA_OK;
+  }
+  if (sms <= 0) {
+    const int rc = current_sm_count(&sms);
+    if (rc != MOA_OK) return rc;
+  }
+  const int64_t units = numel4(B, H, (Nq + kQBlockRows - 1) / kQBlockRows, 1);
+  if (units < 0) return fail(MOA_ERR_INVALID_ARG, "sizes overflow");
+  *sp = plan_splits_auto(units, Nk, sms);
+  return MOA_OK;
+}
+
 }  // namespace
 }  // namespace moa
 
@@ -274,9 +322,29 @@ size_t moa_attn_splitkv_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64
                                         int64_t d_k, int64_t d_v, int dtype, int num_splits) {
   (void)d_k;
   if (dtype != MOA_BF16 || B <= 0 || H <= 0 || N_q <= 0 || N_k <= 0 || d_v <= 0) return 0;
-  const int64_t rows = moa::numel4(B, H, N_q, 1);
-  if (rows < 0) return 0;
-  return moa::splitkv_workspace_bytes(rows, d_v, moa::plan_splits(N_k, num_splits));
+  if (moa::numel4(B, H, N_q, d_v) < 0) return 0;
+  moa::SplitPlan sp;
+  if (moa::choose_plan(B, H, N_q, N_k, num_splits, 0, &sp) != MOA_OK) return 0;
+  return moa::splitkv_workspace_bytes(B * H * N_q, d_v, sp);
+}
+
+int moa_attn_split_plan(int64_t B, int64_t H, int64_t N_q, int64_t N_k, int num_splits,
+                        int sm_count, int* splits, int* key_blocks_per_split,
+                        int64_t* whole_query_blocks) {
+  if (B <= 0 || H <= 0 || N_q <= 0 || N_k <= 0)
+    return moa::fail(MOA_ERR_INVALID_ARG, "sizes must be positive");
+  if (moa::numel4(B, H, N_q, 1) < 0) return moa::fail(MOA_ERR_INVALID_ARG, "sizes overflow");
+  moa::SplitPlan sp;
+  const int rc = moa::choose_plan(B, H, N_q, N_k, num_splits, sm_count, &sp);
+  if (rc != MOA_OK) return rc;
+  const int64_t units = B * H * ((N_q + moa::kQBlockRows - 1) / moa::kQBlockRows);
+  const int64_t n_kt = (N_k + 127) / 128;
+  if (splits) *splits = sp.n_splits;
+  if (key_blocks_per_split)
+    *key_blocks_per_split = int(sp.n_splits > 1 ? sp.kv_per_split : n_kt);
+  if (whole_query_blocks) *whole_query_blocks = sp.n_splits > 1 ? 0 : units;
+  moa::t_last_error[0] = '\0';
+  return MOA_OK;
 }
 
 int moa_attn_fwd_splitkv(const void* Q, const void* K, const void* V, void* O, int64_t B,
@@ -286,10 +354,12 @@ int moa_attn_fwd_splitkv(const void* Q, const void* K, const void* V, void* O, i
   int64_t sz[4];
   int rc = moa::validate(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
   if (rc != MOA_OK) return rc;
-  if (num_splits < 1) return moa::fail(MOA_ERR_INVALID_ARG, "num_splits must be >= 1");
+  if (num_splits < 0) return moa::fail(MOA_ERR_INVALID_ARG, "num_splits must be >= 0");
   if (dtype != MOA_BF16)  // the fp32 path has no split form; it computes the same result whole
     return moa::dispatch(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream);
-  const moa::SplitPlan sp = moa::plan_splits(N_k, num_splits);
+  moa::SplitPlan sp;
+  rc = moa::choose_plan(B, H, N_q, N_k, num_splits, 0, &sp);
+  if (rc != MOA_OK) return rc;
   const size_t need = moa::splitkv_workspace_bytes(B * H * N_q, d_v, sp);
   if (need > 0) {
     if (workspace == nullptr || workspace_bytes < need)
@@ -317,13 +387,19 @@ int moa_attn_fwd_splitkv_noalloc(const void* Q, const void* K, const void* V, vo
   int64_t sz[4];
   int rc = moa::validate(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
   if (rc != MOA_OK) return rc;
-  if (num_splits < 1) return moa::fail(MOA_ERR_INVALID_ARG, "num_splits must be >= 1");
+  if (num_splits < 0) return moa::fail(MOA_ERR_INVALID_ARG, "num_splits must be >= 0");
   if (dtype != MOA_BF16)  // no split form, no scratch: the whole fp32 computation
     return moa::dispatch(Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, dtype, stream);
+  moa::SplitPlan sp;
+  rc = moa::choose_plan(B, H, N_q, N_k, num_splits, 0, &sp);
+  if (rc != MOA_OK) return rc;
+  // The library's own choice never fails for want of scratch: it runs unsplit instead.
+  if (num_splits == MOA_SPLITS_AUTO &&
+      moa::splitkv_workspace_bytes(B * H * N_q, d_v, sp) > moa::kNoallocScratchBytes)
+    sp = moa::SplitPlan{};
   moa::AttnArgs a{Q, K, V, O, B, H, N_q, N_k, d_k, d_v, scale, static_cast<cudaStream_t>(stream)};
   char msg[256] = {0};
-  rc = moa::launch_attn_fwd_bf16_split_noalloc(a, moa::plan_splits(N_k, num_splits), msg,
-                                               sizeof(msg));
+  rc = moa::launch_attn_fwd_bf16_split_noalloc(a, sp, msg, sizeof(msg));
   if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
   moa::t_last_error[0] = '\0';
   return moa::debug_check(stream);

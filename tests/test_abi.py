@@ -4,6 +4,7 @@ import math
 import os
 import re
 
+import numpy as np
 import pytest
 
 import paper_2606_07713_gb300 as pkg
@@ -106,10 +107,61 @@ def test_splitkv_workspace_formula(L):
 
 def test_splitkv_validation_without_gpu(L):
     f = _lib.moa_attn_fwd_splitkv
-    assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 0, 0x500000, 1 << 20, None) == _lib.MOA_ERR_INVALID_ARG
+    assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, -1, 0x500000, 1 << 20, None) == _lib.MOA_ERR_INVALID_ARG
     assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 4, None, 0, None) == _lib.MOA_ERR_INVALID_ARG
     assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 4, 0x500008, 1 << 20, None) == _lib.MOA_ERR_MISALIGNED
     assert f(A, B_, C, D, 1, 1, 8, 1024, 64, 64, 0.1, 1, 4, D, 1 << 20, None) == _lib.MOA_ERR_INVALID_ARG
+
+
+def test_split_plan_of_the_workloads(L):
+    """The library's own split on a 152-SM GPU: only shapes whose query blocks leave SMs idle."""
+    plan = pkg.moa_attn_split_plan
+    auto = pkg.MOA_SPLITS_AUTO
+    # a wave or more of query blocks: nothing is split (the plain kernel runs)
+    assert plan(4, 16, 2048, 2048, auto, 152) == (0, 1, 16, 512)
+    assert plan(2, 32, 8192, 8192, auto, 152) == (0, 1, 64, 2048)
+    assert plan(8, 8, 1024, 4096, auto, 152) == (0, 1, 32, 256)
+    assert plan(1, 152, 256, 4096, auto, 152) == (0, 1, 32, 152)
+    # 16 blocks, 256 key blocks: 9 splits of 29 blocks fill 144 SMs in one round
+    assert plan(1, 16, 256, 32768, auto, 152) == (0, 9, 29, 0)
+    # 8 blocks, 512 key blocks: 16 splits of 32 blocks (at most 32 splits; 19 would not
+    # save 2 % more)
+    assert plan(1, 8, 128, 65536, auto, 152) == (0, 16, 32, 0)
+    # 100 blocks of 16 key blocks: any split needs two rounds; not worth it
+    assert plan(1, 100, 256, 2048, auto, 152) == (0, 1, 16, 100)
+    # too few key blocks to split (each range keeps two)
+    assert plan(1, 2, 256, 300, auto, 152) == (0, 1, 3, 2)
+    # a requested count splits every block
+    assert plan(1, 2, 256, 1000, 3, 152) == (0, 3, 3, 0)
+    assert plan(1, 2, 256, 1000, 1, 152) == (0, 1, 8, 2)
+    assert plan(1, 2, 256, 1000, -1, 152)[0] == _lib.MOA_ERR_INVALID_ARG
+    assert plan(0, 2, 256, 1000, auto, 152)[0] == _lib.MOA_ERR_INVALID_ARG
+    assert plan(1, 2, 256, -5, auto, 152)[0] == _lib.MOA_ERR_INVALID_ARG
+
+
+def test_split_plan_properties(L):
+    """Over random shapes and SM counts, the automatic plan is well formed: it splits only
+    when the query blocks fill less than one wave, every key range is non-empty with at
+    least two key blocks, and the split CTAs are predicted to take at most 0.85 of the time."""
+    rng = np.random.default_rng(7)
+    n_split = 0
+    for _ in range(3000):
+        B, H = int(rng.integers(1, 5)), int(rng.integers(1, 33))
+        Nq, Nk = int(rng.integers(1, 4000)), int(rng.integers(1, 70000))
+        sms = int(rng.integers(1, 300))
+        rc, s, per, whole = pkg.moa_attn_split_plan(B, H, Nq, Nk, pkg.MOA_SPLITS_AUTO, sms)
+        assert rc == 0
+        units = B * H * -(-Nq // 256)
+        n_kt = -(-Nk // 128)
+        if s == 1:
+            assert whole == units and per == n_kt
+            continue
+        n_split += 1
+        assert units < sms and whole == 0
+        assert per >= 2 and (s - 1) * per < n_kt <= s * per and s <= 32
+        rounds = -(-(units * s) // sms)
+        assert rounds * (per / n_kt + 0.08) <= 0.85 + 1e-9
+    assert n_split > 100
 
 
 def test_lse_validation_without_gpu(L):

@@ -63,3 +63,42 @@ def test_splitkv_rejects_small_workspace():
     with pytest.raises(pkg.MoaError) as e:
         pkg.attn_fwd_splitkv(q, k, v, 4, workspace=ws)
     assert e.value.status == _lib.MOA_ERR_INVALID_ARG
+
+
+def _sms():
+    return torch.cuda.get_device_properties(0).multi_processor_count
+
+
+def _auto_case(shape, seed):
+    x = I.make_inputs(I.custom_config(*shape, dtype="bf16", seed=seed))
+    q, k, v = to_device(x)
+    rc, s, per, whole = pkg.moa_attn_split_plan(*shape[:4], pkg.MOA_SPLITS_AUTO, 0)
+    assert rc == 0
+    o = pkg.attn_fwd_splitkv(q, k, v, pkg.MOA_SPLITS_AUTO)
+    torch.cuda.synchronize()
+    pkg.check(pkg.get_device_status())
+    return x, (q, k, v), o, (s, per, whole)
+
+
+@pytest.mark.parametrize("shape", [(1, 4, 64, 4096, 128, 128), (2, 3, 300, 2000, 64, 64),
+                                   (1, 5, 256, 3000, 128, 64)], ids=str)
+def test_splitkv_auto_few_blocks(oracle, shape):
+    """Fewer query blocks than SMs: every block's key axis is split (decode-like shapes, ragged
+    query and key tails)."""
+    x, (q, k, v), o, (s, per, whole) = _auto_case(shape, seed=sum(shape))
+    assert s > 1 and whole == 0
+    assert_close(o.float().cpu().numpy(), oracle.attn(x.q, x.k, x.v, x.scale), "bf16",
+                 f"auto split {shape} splits={s}")
+    need = pkg.moa_attn_splitkv_workspace_bytes(*shape, pkg.MOA_BF16, pkg.MOA_SPLITS_AUTO)
+    assert need == s * shape[0] * shape[1] * shape[2] * (4 * shape[5] + 8)
+
+
+def test_splitkv_auto_no_split_is_the_plain_kernel():
+    """When the plan splits nothing the call is moa_attn_fwd: same bits."""
+    S = _sms()
+    shape = (1, S, 256, 640, 64, 64)
+    x, (q, k, v), o, (s, per, whole) = _auto_case(shape, seed=5)
+    assert s == 1
+    assert torch.equal(o, pkg.attn_fwd(q, k, v))
+    need = pkg.moa_attn_splitkv_workspace_bytes(*shape, pkg.MOA_BF16, pkg.MOA_SPLITS_AUTO)
+    assert need == 0
