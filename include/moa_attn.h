@@ -154,6 +154,38 @@ size_t moa_attn_bwd_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N
                                     int64_t d_v, int dtype);
 
 /*
+ * moa_attn_bwd_fused -- the gradients of moa_attn_bwd from one tile kernel (bf16, d_k = d_v = 64).
+ *
+ * Defines: the same dQ, dK, dV as moa_attn_bwd (paper Stage 5, Section 9).  Each CTA owns a
+ * block of 128 keys and forms the scores and dP of every query block once, computing the three
+ * products dV += W^T dO, dK += dS^T Q and dQ_i = dS_i K from them (5 tile products per block
+ * pair instead of moa_attn_bwd's 7).  The dQ_i of the key blocks are summed in an fp32
+ * accumulator in the workspace with atomic additions, then scaled and rounded to bf16.
+ * Arguments, layouts, alignment and overlap rules: those of moa_attn_bwd, with
+ * dtype MOA_BF16 and d_k = d_v = 64 only, and a workspace of at least
+ * moa_attn_bwd_fused_workspace_bytes(...) bytes.
+ * Reproducibility: dK and dV are bitwise reproducible; the order of the fp32 additions into dQ
+ * varies between runs, so dQ may differ in its last bits from run to run (moa_attn_bwd's dQ
+ * does not).
+ * Errors: those of moa_attn_bwd; MOA_ERR_UNSUPPORTED_DTYPE for fp32, MOA_ERR_UNSUPPORTED_SHAPE
+ * for other head dimensions.
+ * Behaviour: asynchronous; three kernel launches on `stream` (per-row D and LSE with the
+ * accumulator zeroed, the tile kernel, the dQ conversion).  Allocates nothing.
+ */
+int moa_attn_bwd_fused(const void* Q, const void* K, const void* V, const void* O,
+                       const void* dO, const float* LSE, void* dQ, void* dK, void* dV, int64_t B,
+                       int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v, float scale,
+                       int dtype, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * moa_attn_bwd_fused_workspace_bytes -- scratch bytes moa_attn_bwd_fused needs: (2 + d_k) fp32
+ * values per (b, h) and query row, rows padded to a multiple of 128 (0 unless dtype is
+ * MOA_BF16 and d_k = d_v = 64, or for sizes < 1).
+ */
+size_t moa_attn_bwd_fused_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k,
+                                          int64_t d_k, int64_t d_v, int dtype);
+
+/*
  * moa_qkv_proj -- the input projections Q = X W_Q, K = X W_K, V = X W_V in one pass.
  *
  * Defines: paper Section 4.1 (the problem setup: Q, K, V are the input sequence X projected

@@ -18,7 +18,8 @@ from ._lib import (MOA_BF16, MOA_FP32, MoaError, check, lib, moa_attn_dnf_bytes,
                    moa_get_device_status, moa_last_error, moa_selftest_wait_timeout,
                    moa_attn_fwd_splitkv, moa_attn_splitkv_workspace_bytes, moa_attn_fwd_lse,
                    moa_attn_bwd, moa_attn_bwd_workspace_bytes, moa_qkv_proj,
-                   moa_attn_split_plan, MOA_SPLITS_AUTO)
+                   moa_attn_split_plan, MOA_SPLITS_AUTO, moa_attn_bwd_fused,
+                   moa_attn_bwd_fused_workspace_bytes)
 
 __all__ = ["attn_fwd", "attn_fwd_staged", "get_device_status", "attn_flops", "dnf_bytes",
            "MOA_FP32", "MOA_BF16", "MoaError", "moa_attn_fwd", "moa_attn_fwd_staged",
@@ -26,7 +27,8 @@ __all__ = ["attn_fwd", "attn_fwd_staged", "get_device_status", "attn_flops", "dn
            "moa_attn_version", "moa_selftest_wait_timeout", "attn_fwd_splitkv",
            "moa_attn_fwd_splitkv", "moa_attn_splitkv_workspace_bytes", "attn_fwd_lse",
            "moa_attn_fwd_lse", "attn_bwd", "moa_attn_bwd", "moa_attn_bwd_workspace_bytes",
-           "qkv_proj", "moa_qkv_proj", "moa_attn_split_plan", "MOA_SPLITS_AUTO"]
+           "qkv_proj", "moa_qkv_proj", "moa_attn_split_plan", "MOA_SPLITS_AUTO",
+           "moa_attn_bwd_fused", "moa_attn_bwd_fused_workspace_bytes"]
 
 
 def _dtype_code(t) -> int:
@@ -107,9 +109,11 @@ def attn_fwd_lse(q, k, v, scale: float | None = None, out=None, lse=None, stream
     return out, lse
 
 
-def attn_bwd(q, k, v, o, lse, do, scale: float | None = None, workspace=None, stream=None):
+def attn_bwd(q, k, v, o, lse, do, scale: float | None = None, workspace=None, stream=None,
+             fused: bool = False):
     """(dQ, dK, dV) for O = softmax(scale q k^T) v given dO = dL/dO, from the forward's o and lse
-    (attn_fwd_lse).  bf16 CUDA tensors [B, H, N, d]; lse float32 [B, H, N_q]."""
+    (attn_fwd_lse).  CUDA tensors [B, H, N, d]; lse float32 [B, H, N_q].  fused=True runs
+    moa_attn_bwd_fused (bf16, d_k = d_v = 64; dQ summed with atomics)."""
     import torch
     for t in (q, k, v, o, do, lse):
         if not t.is_cuda or not t.is_contiguous():
@@ -127,15 +131,17 @@ def attn_bwd(q, k, v, o, lse, do, scale: float | None = None, workspace=None, st
     dq = torch.empty_like(q)
     dkk = torch.empty_like(k)
     dvv = torch.empty_like(v)
-    need = moa_attn_bwd_workspace_bytes(B, H, Nq, Nk, dk, dv, code)
+    wsb = moa_attn_bwd_fused_workspace_bytes if fused else moa_attn_bwd_workspace_bytes
+    call = moa_attn_bwd_fused if fused else moa_attn_bwd
+    need = wsb(B, H, Nq, Nk, dk, dv, code)
     if workspace is None:
         workspace = torch.empty(max(need, 16), dtype=torch.uint8, device=q.device)
     with torch.cuda.device(q.device):
         s = stream if stream is not None else torch.cuda.current_stream(q.device)
-        check(moa_attn_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(), do.data_ptr(),
-                           lse.data_ptr(), dq.data_ptr(), dkk.data_ptr(), dvv.data_ptr(), B, H, Nq,
-                           Nk, dk, dv, float(scale), code, workspace.data_ptr(), workspace.numel(),
-                           s.cuda_stream))
+        check(call(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(), do.data_ptr(),
+                   lse.data_ptr(), dq.data_ptr(), dkk.data_ptr(), dvv.data_ptr(), B, H, Nq, Nk, dk,
+                   dv, float(scale), code, workspace.data_ptr(), workspace.numel(),
+                   s.cuda_stream))
     return dq, dkk, dvv
 
 

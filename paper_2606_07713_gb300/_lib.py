@@ -44,6 +44,11 @@ SIGNATURES = {
                                     ctypes.c_size_t, _VP]),
     "moa_attn_bwd_workspace_bytes": (ctypes.c_size_t, [_I64, _I64, _I64, _I64, _I64, _I64,
                                                        ctypes.c_int]),
+    "moa_attn_bwd_fused": (ctypes.c_int, [_VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _I64, _I64,
+                                          _I64, _I64, _I64, _I64, ctypes.c_float, ctypes.c_int,
+                                          _VP, ctypes.c_size_t, _VP]),
+    "moa_attn_bwd_fused_workspace_bytes": (ctypes.c_size_t, [_I64, _I64, _I64, _I64, _I64, _I64,
+                                                             ctypes.c_int]),
     "moa_qkv_proj": (ctypes.c_int, [_VP, _VP, _VP, _VP, _VP, _I64, _I64, _I64, _I64, _I64, _I64,
                                     ctypes.c_int, _VP]),
     "moa_attn_fwd_staged": (ctypes.c_int, [_VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _I64, _I64,
@@ -124,6 +129,16 @@ def moa_attn_bwd(Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v, scal
 
 def moa_attn_bwd_workspace_bytes(B, H, N_q, N_k, d_k, d_v, dtype) -> int:
     return lib().moa_attn_bwd_workspace_bytes(B, H, N_q, N_k, d_k, d_v, dtype)
+
+
+def moa_attn_bwd_fused(Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v, scale, dtype,
+                       workspace, workspace_bytes, stream) -> int:
+    return lib().moa_attn_bwd_fused(Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v,
+                                    scale, dtype, workspace, workspace_bytes, stream)
+
+
+def moa_attn_bwd_fused_workspace_bytes(B, H, N_q, N_k, d_k, d_v, dtype) -> int:
+    return lib().moa_attn_bwd_fused_workspace_bytes(B, H, N_q, N_k, d_k, d_v, dtype)
 
 
 def moa_qkv_proj(X, W, Q, K, V, B, N, d_model, H, d_k, d_v, dtype, stream) -> int:

@@ -727,6 +727,27 @@ bool encode_bf16_map_box(CUtensorMap* map, const void* base, int64_t BH, int64_t
   return true;
 }
 
+// 3-D map over a contiguous fp32 [BH, N, d] tensor; box = box_cols columns (32: one 128-byte
+// swizzle row) x box_rows rows x 1 slice, 128-byte swizzle.
+bool encode_f32_map_sw128(CUtensorMap* map, const void* base, int64_t BH, int64_t N, int64_t d,
+                          int box_cols, int box_rows, char* msg, size_t msglen) {
+  EncodeTiledFn enc = get_encode_fn(msg, msglen);
+  if (!enc) return false;
+  const cuuint64_t dims[3] = {cuuint64_t(d), cuuint64_t(N), cuuint64_t(BH)};
+  const cuuint64_t strides[2] = {cuuint64_t(d * 4), cuuint64_t(N * d * 4)};
+  const cuuint32_t box[3] = {cuuint32_t(box_cols), cuuint32_t(box_rows), 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(base), dims, strides,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    snprintf(msg, msglen, "cuTensorMapEncodeTiled failed (%d) for fp32 [%lld,%lld,%lld]", int(r),
+             (long long)BH, (long long)N, (long long)d);
+    return false;
+  }
+  return true;
+}
+
 namespace {
 
 template <int DK, int DV>

@@ -62,6 +62,10 @@ int launch_attn_fwd_bf16_split_noalloc(const AttnArgs& a, const SplitPlan& sp, c
 // swizzle, rows past N of a slice read as zero.  False (and a message) on failure.
 bool encode_bf16_map(CUtensorMap* map, const void* base, int64_t BH, int64_t N, int64_t d,
                      char* msg, size_t msglen);
+// Map over a contiguous fp32 [BH, N, d] tensor: box of box_cols columns (at most 32) x box_rows
+// rows, 128-byte swizzle.
+bool encode_f32_map_sw128(CUtensorMap* map, const void* base, int64_t BH, int64_t N, int64_t d,
+                          int box_cols, int box_rows, char* msg, size_t msglen);
 // Same with a box of box_rows rows (64 columns, 128-byte swizzle).
 bool encode_bf16_map_box(CUtensorMap* map, const void* base, int64_t BH, int64_t N, int64_t d,
                          int box_rows, char* msg, size_t msglen);
@@ -100,6 +104,10 @@ struct BwdArgs {
 // log-sum-exp (bf16 path: in log2 units, negated), fp32.
 size_t bwd_workspace_bytes(int64_t B, int64_t H, int64_t Nq);
 int launch_attn_bwd_bf16(const BwdArgs& a, char* msg, size_t msglen);
+// One kernel for dK, dV and dQ (bf16, d_k = d_v = 64); the workspace adds an fp32 dQ
+// accumulator of padded rows x d_k after the two per-row vectors.
+size_t bwd_fused_workspace_bytes(int64_t B, int64_t H, int64_t Nq, int64_t dk);
+int launch_attn_bwd_bf16_fused(const BwdArgs& a, char* msg, size_t msglen);
 // fp32 backward on CUDA cores; same workspace layout (LSE instead of -LSE log2 e in the first half).
 int launch_attn_bwd_f32(const BwdArgs& a, char* msg, size_t msglen);
 // Reads and clears the status word of the backward kernels' bounded waits (after a sync).

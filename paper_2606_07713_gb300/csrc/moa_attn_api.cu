@@ -215,6 +215,59 @@ int choose_plan(int64_t B, int64_t H, int64_t Nq, int64_t Nk, int num_splits, in
   return MOA_OK;
 }
 
+// Validation and dispatch of the two backward entry points.
+int bwd_call(const void* Q, const void* K, const void* V, const void* O, const void* dO,
+             const float* LSE, void* dQ, void* dK, void* dV, int64_t B, int64_t H, int64_t N_q,
+             int64_t N_k, int64_t d_k, int64_t d_v, float scale, int dtype, void* workspace,
+             size_t workspace_bytes, void* stream, bool fused) {
+  if (!dO || !LSE || !dQ || !dK || !dV)
+    return fail(MOA_ERR_INVALID_ARG, "null pointer among dO, LSE, dQ, dK, dV");
+  int64_t sz[4];
+  int rc = validate(Q, K, V, const_cast<void*>(O), B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
+  if (rc != MOA_OK) return rc;
+  if (fused && dtype != MOA_BF16)
+    return fail(MOA_ERR_UNSUPPORTED_DTYPE, "the fused backward takes bf16 tensors only");
+  if (fused && (d_k != 64 || d_v != 64))
+    return fail(MOA_ERR_UNSUPPORTED_SHAPE, "the fused backward needs d_k = d_v = 64; got %lld, %lld",
+                (long long)d_k, (long long)d_v);
+  const void* al[5] = {dO, dQ, dK, dV, workspace};
+  for (const void* p : al)
+    if (reinterpret_cast<uintptr_t>(p) % 16 != 0)
+      return fail(MOA_ERR_MISALIGNED, "pointer %p is not 16-byte aligned", p);
+  if (reinterpret_cast<uintptr_t>(LSE) % 4 != 0)
+    return fail(MOA_ERR_MISALIGNED, "LSE pointer is not 4-byte aligned");
+  if (fused && numel4(B, H, N_q + 127, 2 + d_k) < 0)
+    return fail(MOA_ERR_INVALID_ARG, "sizes overflow");
+  const size_t need = fused ? bwd_fused_workspace_bytes(B, H, N_q, d_k)
+                            : bwd_workspace_bytes(B, H, N_q);
+  if (workspace == nullptr || workspace_bytes < need)
+    return fail(MOA_ERR_INVALID_ARG, "workspace too small: need %zu bytes, got %zu", need,
+                workspace == nullptr ? size_t(0) : workspace_bytes);
+  // Read-only: Q, K, V, O, dO, LSE.  Written: dQ, dK, dV, workspace (no two may overlap, and
+  // none may overlap a read-only buffer).
+  const void* ro[6] = {Q, K, V, O, dO, LSE};
+  const int64_t rosz[6] = {sz[0], sz[1], sz[2], sz[3], sz[3], B * H * N_q * 4};
+  const void* wr[4] = {dQ, dK, dV, workspace};
+  const int64_t wrsz[4] = {sz[0], sz[1], sz[2], int64_t(need)};
+  for (int i = 0; i < 4; ++i) {
+    for (int j = 0; j < 6; ++j)
+      if (overlaps(wr[i], wrsz[i], ro[j], rosz[j]))
+        return fail(MOA_ERR_INVALID_ARG, "an output or the workspace overlaps an input");
+    for (int j = i + 1; j < 4; ++j)
+      if (overlaps(wr[i], wrsz[i], wr[j], wrsz[j]))
+        return fail(MOA_ERR_INVALID_ARG, "outputs or the workspace overlap each other");
+  }
+  BwdArgs a{Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v, scale, workspace,
+            static_cast<cudaStream_t>(stream)};
+  char msg[256] = {0};
+  rc = fused ? launch_attn_bwd_bf16_fused(a, msg, sizeof(msg))
+             : dtype == MOA_BF16 ? launch_attn_bwd_bf16(a, msg, sizeof(msg))
+                                 : launch_attn_bwd_f32(a, msg, sizeof(msg));
+  if (rc != MOA_OK) return fail(rc, "%s", msg);
+  t_last_error[0] = '\0';
+  return debug_check(stream);
+}
+
 }  // namespace
 }  // namespace moa
 
@@ -419,43 +472,24 @@ int moa_attn_bwd(const void* Q, const void* K, const void* V, const void* O, con
                  const float* LSE, void* dQ, void* dK, void* dV, int64_t B, int64_t H,
                  int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v, float scale, int dtype,
                  void* workspace, size_t workspace_bytes, void* stream) {
-  if (!dO || !LSE || !dQ || !dK || !dV)
-    return moa::fail(MOA_ERR_INVALID_ARG, "null pointer among dO, LSE, dQ, dK, dV");
-  int64_t sz[4];
-  int rc = moa::validate(Q, K, V, const_cast<void*>(O), B, H, N_q, N_k, d_k, d_v, scale, dtype, sz);
-  if (rc != MOA_OK) return rc;
-  const void* al[5] = {dO, dQ, dK, dV, workspace};
-  for (const void* p : al)
-    if (reinterpret_cast<uintptr_t>(p) % 16 != 0)
-      return moa::fail(MOA_ERR_MISALIGNED, "pointer %p is not 16-byte aligned", p);
-  if (reinterpret_cast<uintptr_t>(LSE) % 4 != 0)
-    return moa::fail(MOA_ERR_MISALIGNED, "LSE pointer is not 4-byte aligned");
-  const size_t need = moa::bwd_workspace_bytes(B, H, N_q);
-  if (workspace == nullptr || workspace_bytes < need)
-    return moa::fail(MOA_ERR_INVALID_ARG, "workspace too small: need %zu bytes, got %zu", need,
-                     workspace == nullptr ? size_t(0) : workspace_bytes);
-  // Read-only: Q, K, V, O, dO, LSE.  Written: dQ, dK, dV, workspace (no two may overlap, and
-  // none may overlap a read-only buffer).
-  const void* ro[6] = {Q, K, V, O, dO, LSE};
-  const int64_t rosz[6] = {sz[0], sz[1], sz[2], sz[3], sz[3], B * H * N_q * 4};
-  const void* wr[4] = {dQ, dK, dV, workspace};
-  const int64_t wrsz[4] = {sz[0], sz[1], sz[2], int64_t(need)};
-  for (int i = 0; i < 4; ++i) {
-    for (int j = 0; j < 6; ++j)
-      if (moa::overlaps(wr[i], wrsz[i], ro[j], rosz[j]))
-        return moa::fail(MOA_ERR_INVALID_ARG, "an output or the workspace overlaps an input");
-    for (int j = i + 1; j < 4; ++j)
-      if (moa::overlaps(wr[i], wrsz[i], wr[j], wrsz[j]))
-        return moa::fail(MOA_ERR_INVALID_ARG, "outputs or the workspace overlap each other");
-  }
-  moa::BwdArgs a{Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v, scale, workspace,
-                 static_cast<cudaStream_t>(stream)};
-  char msg[256] = {0};
-  rc = dtype == MOA_BF16 ? moa::launch_attn_bwd_bf16(a, msg, sizeof(msg))
-                         : moa::launch_attn_bwd_f32(a, msg, sizeof(msg));
-  if (rc != MOA_OK) return moa::fail(rc, "%s", msg);
-  moa::t_last_error[0] = '\0';
-  return moa::debug_check(stream);
+  return moa::bwd_call(Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v, scale, dtype,
+                       workspace, workspace_bytes, stream, false);
+}
+
+int moa_attn_bwd_fused(const void* Q, const void* K, const void* V, const void* O,
+                       const void* dO, const float* LSE, void* dQ, void* dK, void* dV, int64_t B,
+                       int64_t H, int64_t N_q, int64_t N_k, int64_t d_k, int64_t d_v, float scale,
+                       int dtype, void* workspace, size_t workspace_bytes, void* stream) {
+  return moa::bwd_call(Q, K, V, O, dO, LSE, dQ, dK, dV, B, H, N_q, N_k, d_k, d_v, scale, dtype,
+                       workspace, workspace_bytes, stream, true);
+}
+
+size_t moa_attn_bwd_fused_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N_k,
+                                          int64_t d_k, int64_t d_v, int dtype) {
+  (void)N_k;
+  if (dtype != MOA_BF16 || d_k != 64 || d_v != 64 || B < 1 || H < 1 || N_q < 1) return 0;
+  if (moa::numel4(B, H, N_q + 127, 2 + d_k) < 0) return 0;
+  return moa::bwd_fused_workspace_bytes(B, H, N_q, d_k);
 }
 
 int moa_qkv_proj(const void* X, const void* W, void* Q, void* K, void* V, int64_t B, int64_t N,

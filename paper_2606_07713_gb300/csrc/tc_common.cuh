@@ -19,6 +19,10 @@ __host__ __device__ constexpr uint32_t make_idesc(int M, int N, bool b_mn_major)
   return (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | ((b_mn_major ? 1u : 0u) << 16) |
          (uint32_t(N >> 3) << 17) | (uint32_t(M >> 4) << 24);
 }
+// Same with the A operand (from shared memory) MN-major as well (bit 15: A transposed).
+__host__ __device__ constexpr uint32_t make_idesc_a_mn(int M, int N, bool b_mn_major) {
+  return make_idesc(M, N, b_mn_major) | (1u << 15);
+}
 
 // Shared-memory matrix descriptor, 128-byte swizzle (layout code 2 in bits 61-63), version 1
 // (bits 46-47).  Start address, leading and stride byte offsets in 16-byte units.

@@ -176,6 +176,26 @@ def test_lse_validation_without_gpu(L):
     assert f(A, B_, C, D, E, 1, 1, 8, 8, 96, 64, 0.125, 1, None) == _lib.MOA_ERR_UNSUPPORTED_SHAPE
 
 
+def test_bwd_fused_workspace_formula_and_validation(L):
+    ws = pkg.moa_attn_bwd_fused_workspace_bytes
+    assert ws(2, 3, 200, 300, 64, 64, pkg.MOA_BF16) == 2 * 3 * 256 * 4 * (2 + 64)
+    assert ws(1, 1, 128, 5, 64, 64, pkg.MOA_BF16) == 128 * 4 * 66
+    assert ws(1, 1, 128, 5, 128, 64, pkg.MOA_BF16) == 0     # d_k = d_v = 64 only
+    assert ws(1, 1, 128, 5, 64, 64, pkg.MOA_FP32) == 0
+    assert ws(0, 1, 128, 5, 64, 64, pkg.MOA_BF16) == 0
+    f = _lib.moa_attn_bwd_fused
+    E = 0x600000
+    args = (1, 1, 128, 128, 64, 64, 0.125, 1)
+    W = 0x700000
+    need = ws(1, 1, 128, 128, 64, 64, pkg.MOA_BF16)
+    # workspace too small, misaligned, overlapping; other head sizes; fp32
+    assert f(A, B_, C, D, E, 0x680000, 0x800000, 0x810000, 0x820000, *args, W, need - 16, None) == _lib.MOA_ERR_INVALID_ARG
+    assert f(A, B_, C, D, E, 0x680000, 0x800000, 0x810000, 0x820000, *args, W + 8, need, None) == _lib.MOA_ERR_MISALIGNED
+    assert f(A, B_, C, D, E, 0x680000, 0x800000, 0x810000, 0x820000, *args, A, need, None) == _lib.MOA_ERR_INVALID_ARG
+    assert f(A, B_, C, D, E, 0x680000, 0x800000, 0x810000, 0x820000, 1, 1, 128, 128, 128, 128, 0.125, 1, W, 1 << 24, None) == _lib.MOA_ERR_UNSUPPORTED_SHAPE
+    assert f(A, B_, C, D, E, 0x680000, 0x800000, 0x810000, 0x820000, 1, 1, 128, 128, 64, 64, 0.125, 0, W, 1 << 24, None) == _lib.MOA_ERR_UNSUPPORTED_DTYPE
+
+
 def test_bwd_workspace_formula(L):
     ws = pkg.moa_attn_bwd_workspace_bytes
     assert ws(2, 3, 200, 300, 64, 64, pkg.MOA_BF16) == 2 * 2 * 3 * 256 * 4
