@@ -375,8 +375,12 @@ def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
     g, gbits = I.make_grad_output(cfg)
     q, k, v, do = (to_device_bf16(b, dev) for b in (x.q_bits, x.k_bits, x.v_bits, gbits))
     o, lse = pkg.attn_fwd_lse(q, k, v, cfg.scale)
-    ws = torch.empty(pkg.moa_attn_bwd_workspace_bytes(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v,
-                                                      pkg.MOA_BF16), dtype=torch.uint8, device=dev)
+    # d_k = d_v = 64: the one-kernel backward (5 tile products); otherwise the three-kernel one.
+    # --bwd-path picks one explicitly.
+    fused = args.bwd_path == "fused" or (args.bwd_path == "auto" and s.d_k == 64 and s.d_v == 64)
+    wsb = pkg.moa_attn_bwd_fused_workspace_bytes if fused else pkg.moa_attn_bwd_workspace_bytes
+    ws = torch.empty(max(16, wsb(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v, pkg.MOA_BF16)),
+                     dtype=torch.uint8, device=dev)
     host = [t.cpu().pin_memory() for t in (q, k, v, o, do, lse)]
     host_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in (q, k, v)]
     flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
@@ -390,7 +394,7 @@ def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
 
     for _ in range(args.warmup):
         flush.zero_()
-        pkg.attn_bwd(q, k, v, o, lse, do, cfg.scale, workspace=ws)
+        pkg.attn_bwd(q, k, v, o, lse, do, cfg.scale, workspace=ws, fused=fused)
     torch.cuda.synchronize(dev)
     pkg.check(pkg.get_device_status())
     sampler = ClockSampler(local)
@@ -402,7 +406,7 @@ def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
     for i in range(args.steps):
         flush.zero_()
         ev[i][0].record(stream)
-        pkg.attn_bwd(q, k, v, o, lse, do, cfg.scale, workspace=ws, stream=stream)
+        pkg.attn_bwd(q, k, v, o, lse, do, cfg.scale, workspace=ws, stream=stream, fused=fused)
         ev[i][1].record(stream)
     barrier()
     kern_ms = [a.elapsed_time(b) for a, b in ev]
@@ -418,7 +422,8 @@ def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
         ev2[i][0].record(stream)
         for d_, h_ in zip(dev_in, host):
             d_.copy_(h_, non_blocking=True)
-        grads = pkg.attn_bwd(*dev_in[:4], dev_in[5], dev_in[4], cfg.scale, workspace=ws, stream=stream)
+        grads = pkg.attn_bwd(*dev_in[:4], dev_in[5], dev_in[4], cfg.scale, workspace=ws,
+                             stream=stream, fused=fused)
         for h_, d_ in zip(host_out, grads):
             h_.copy_(d_, non_blocking=True)
         ev2[i][1].record(stream)
@@ -440,13 +445,16 @@ def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
             "data": "synthetic: seeded splitmix64 + Box-Muller inputs and dO of the workload's shape",
             "config": dict(workload_desc(cfg), **{
                 "workload": workload_desc(cfg)["workload"].replace("SDPA fwd", "SDPA bwd"),
-                "pass": "backward (moa_attn_bwd)"}),
+                "pass": "backward (moa_attn_bwd_fused)" if fused else "backward (moa_attn_bwd)",
+                "tile_products_executed_per_block_pair": 5 if fused else 7}),
             "compulsory_bytes": bwd_bytes(s),
             "roofline": {
                 "bound": "tensor", "achieved": round(achieved, 2), "peak": peak,
                 "peak_source": f"{peak_src} bf16_tflops (burst; call timed alone)",
                 "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": None,
-                "kernel": "moa_attn_bwd: attn_bwd_pre + attn_bwd_dkdv + attn_bwd_dq (one call)",
+                "kernel": ("moa_attn_bwd_fused: attn_bwd_pre + attn_bwd_fused + attn_bwd_dq_convert"
+                           if fused else
+                           "moa_attn_bwd: attn_bwd_pre + attn_bwd_dkdv + attn_bwd_dq") + " (one call)",
             },
             "e2e": {
                 "value": round(whole_job_tflops(flops, args.steps, world, e2e_ms), 2),
@@ -775,6 +783,9 @@ def main():
     ap.add_argument("--workload", type=int, default=DEFAULT_WORKLOAD, choices=sorted(I.CONFIGS))
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle time for the cpu_baseline sample")
+    ap.add_argument("--bwd-path", choices=["auto", "fused", "split"], default="auto",
+                    help="backward kernels: fused (one tile kernel, d_k = d_v = 64), split (dK/dV "
+                         "and dQ kernels), auto (fused where it applies)")
     ap.add_argument("--pass", dest="which", choices=["fwd", "bwd", "qkv"], default="fwd",
                     help="time the forward (default), the backward pass or the QKV projection")
     ap.add_argument("--shape", default=None,

@@ -950,7 +950,7 @@ attn_bwd_fused_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
         mma_commit(dp_full);
       };
       auto stage = [&](int st) { return sStage + st * C::kStageBytes; };
-      // Issue order S(0) dP(0) | dV(0) S(1) dK(0) dQ(0) dP(1) | dV(1) S(2) dK(1) dQ(1) dP(2) | ...
+      // Issue order S(0) dP(0) | dV(0) S(1) dK(0) dP(1) dQ(0) | dV(1) S(2) dK(1) dP(2) dQ(1) | ...
       bool ok = wait_bounded(kv_full, 0, wc) && wait_bounded(full_bar(0), 0, wc);
       if (ok) {
         tc_fence_after_sync();
@@ -992,6 +992,8 @@ attn_bwd_fused_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
                      make_sdesc_sw128(sQ + kk * 2048, kPanelBytes, 1024), kIdescDK,
                      (kk > 0 || i > 0) ? 1u : 0u);
         }
+        // dP(i+1) before dQ(i): the compute warps wait for it next.
+        if (more) issue_dp(stage(slot) + C::kQBytes);
         // dQ_i = dS K into TMEM buffer i % 2 (free once the compute warps read dQ_{i-2}):
         // A = the same dS^T tile read MN-major (query rows contiguous: 16 keys per step,
         // 64-query panels kPanelBytes apart), B = K tile MN-major.
@@ -1010,7 +1012,6 @@ attn_bwd_fused_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
         mma_commit(dq_full(b));
         mma_commit(ds_free);        // dK(i) and dQ(i) have read dS(i)
         mma_commit(empty_bar(st));  // dV(i) read dO(i), dK(i) read Q(i)
-        if (more) issue_dp(stage(slot) + C::kQBytes);
       }
       // Always signal once everything issued has completed, so that TMEM is quiescent before
       // it is freed even on the abort path.
