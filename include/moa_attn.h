@@ -217,7 +217,8 @@ int moa_qkv_proj(const void* X, const void* W, void* Q, void* K, void* V, int64_
  * hV (host memory, ideally page-locked) into the caller's device buffers dQ,
  * dK, dV, runs the attention on them and copies dO back into hO.  The (b, h)
  * problems are independent (Remark in Section 4.2), so the call is pipelined
- * over up to four contiguous ranges of heads: the copies of range c+1 into the
+ * over contiguous ranges of heads (2 to 8 of them, about 16 MiB of inputs each,
+ * at most one per (b, h)): the copies of range c+1 into the
  * device run on a library-owned side stream while the kernel of range c runs on
  * `stream`, and each range's output goes back on a second side stream.  Work
  * already queued on `stream` completes before the first copy starts, and

@@ -165,12 +165,18 @@ int dispatch(const void* Q, const void* K, const void* V, void* O, int64_t B, in
 // Side streams and events of the pipelined staged call, one set per device, created on the
 // device's first staged call.  The mutex is held while a call enqueues its work, so the events
 // of two concurrent calls never interleave.
-constexpr int kStageChunks = 4;
+// Head ranges of the staged call: about kStageChunkBytes of inputs each, 2 to kMaxStageChunks
+// of them (measured on a GB300: 4x16x2048^2 d=64, 50 MB of inputs, is fastest with 4 ranges,
+// 191 TFLOP/s end to end vs 183 with 2 and 173 with 8; 2x32x8192^2 d=128, 403 MB, with 6 to 8,
+// 905 vs 830 with 4: more ranges shorten the pipeline's fill and drain, smaller ones copy less
+// efficiently).
+constexpr int kMaxStageChunks = 8;
+constexpr int64_t kStageChunkBytes = int64_t(16) << 20;
 constexpr int kMaxDevices = 64;
 struct StagePipe {
   cudaStream_t copy_in = nullptr, copy_out = nullptr;
   cudaEvent_t start = nullptr, end = nullptr;
-  cudaEvent_t in_done[kStageChunks] = {}, kern_done[kStageChunks] = {};
+  cudaEvent_t in_done[kMaxStageChunks] = {}, kern_done[kMaxStageChunks] = {};
   bool ready = false;
 };
 StagePipe g_pipes[kMaxDevices];
@@ -181,7 +187,7 @@ cudaError_t make_pipe(StagePipe& p) {
   if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p.copy_out, cudaStreamNonBlocking);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p.start, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p.end, cudaEventDisableTiming);
-  for (int c = 0; e == cudaSuccess && c < kStageChunks; ++c) {
+  for (int c = 0; e == cudaSuccess && c < kMaxStageChunks; ++c) {
     e = cudaEventCreateWithFlags(&p.in_done[c], cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p.kern_done[c], cudaEventDisableTiming);
   }
@@ -320,10 +326,13 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
   if (!p.ready && (e = moa::make_pipe(p)) != cudaSuccess)
     return moa::fail(MOA_ERR_CUDA, "staged pipeline set-up: %s", cudaGetErrorString(e));
   const int64_t BH = B * H;
-  const int chunks = int(BH < moa::kStageChunks ? BH : moa::kStageChunks);
-  const int64_t per = (BH + chunks - 1) / chunks;
   const int64_t elt = dtype == MOA_FP32 ? 4 : 2;
   const int64_t row_bytes[4] = {N_q * d_k * elt, N_k * d_k * elt, N_k * d_v * elt, N_q * d_v * elt};
+  const int64_t in_bytes = sz[0] + sz[1] + sz[2];
+  int64_t want = (in_bytes + moa::kStageChunkBytes - 1) / moa::kStageChunkBytes;
+  want = want < 2 ? 2 : (want > moa::kMaxStageChunks ? moa::kMaxStageChunks : want);
+  const int chunks = int(BH < want ? BH : want);
+  const int64_t per = (BH + chunks - 1) / chunks;
   const void* src[3] = {hQ, hK, hV};
   void* dst[3] = {dQ, dK, dV};
   auto chk = [&](cudaError_t err, const char* what) {
