@@ -69,6 +69,24 @@ def test_fused_bwd_parity(oracle, shape):
         assert err <= BF16_TOL, f"{shape} {name}: max|g-g_ref|/max|g_ref| = {err:.3e}"
 
 
+@pytest.mark.parametrize("scale", [-0.3, 2.0 / 8, 0.0])
+def test_fused_bwd_other_scales(oracle, scale):
+    """A negative scale (the maximum of the scaled scores is then at the smallest dot product),
+    a larger one, and zero (uniform weights: dQ = dK = 0, dV = the column mean of dO)."""
+    cfg = I.custom_config(1, 2, 260, 700, 64, 64, dtype="bf16", seed=77)
+    x = I.make_inputs(cfg)
+    g, gb = I.make_grad_output(cfg)
+    got = [t.float().cpu().numpy() for t in grads(x, gb, True, scale=scale)]
+    ref = oracle.attn_bwd(x.q, x.k, x.v, g, scale)
+    for name, a, b in zip(("dQ", "dK", "dV"), got, ref):
+        assert np.all(np.isfinite(a)), f"scale {scale} {name}"
+        if np.max(np.abs(b)) == 0.0:
+            assert np.max(np.abs(a)) <= 1e-3, f"scale {scale} {name}: {np.max(np.abs(a)):.3e} for 0"
+            continue
+        err = rel_err(a, b)
+        assert err <= BF16_TOL, f"scale {scale} {name}: {err:.3e}"
+
+
 def test_fused_matches_three_kernel_backward():
     """dK and dV: the same products in the same order of accumulation inside each CTA, so the
     same bits; dQ: the same products summed in another order (fp32), within bf16 rounding."""
