@@ -10,9 +10,7 @@
 //
 // Tiling: persistent CTAs (one per SM) walk the 128-token x 256-column tiles of C; d in steps
 // of 64 through a 4-stage TMA ring (X tile 128 x 64 K-major, W tile 64 x 256 MN-major: the
-// weights are read as stored).  When the tiles fill at most a quarter of the last round of CTAs,
-// each tile of that round is cut into 4 pieces of 64 columns, so that the round takes about a
-// quarter of a tile's time instead of a whole one.  Two 256-column TMEM accumulators alternate between tiles, so the
+// weights are read as stored).  Two 256-column TMEM accumulators alternate between tiles, so the
 // epilogue of one tile overlaps the main loop of the next.  Warps: 0 TMA, 1 TMEM allocation +
 // MMA issue, 2-5 epilogue (warp w owns TMEM lanes 32*(w%4): the 128 token rows).  Waits are
 // bounded (status word g_moa_proj_status).
@@ -63,35 +61,13 @@ struct ProjDims {
   int ncol;     // 2 H dk + H dv
   int n_ktiles; // ceil(d / 64)
   int n_ntiles; // ceil(ncol / 256)
-  int n_full;   // work items [0, n_full) are whole tiles
-  int pieces;   // each later tile is cut into `pieces` items of 256 / pieces columns
 };
-
-// Work item -> (first token row, first column, columns).
-struct ProjItem {
-  int m0, c0, width;
-};
-__device__ __forceinline__ ProjItem proj_item(const ProjDims& p, int item) {
-  ProjItem w;
-  int t = item;
-  w.width = kBN;
-  int piece = 0;
-  if (item >= p.n_full) {
-    const int r = item - p.n_full;
-    t = p.n_full + r / p.pieces;
-    piece = r % p.pieces;
-    w.width = kBN / p.pieces;
-  }
-  w.m0 = (t / p.n_ntiles) * kBM;
-  w.c0 = (t % p.n_ntiles) * kBN + piece * w.width;
-  return w;
-}
 
 __global__ void __launch_bounds__(kThreads, 1)
 qkv_proj_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmX,
                         const __grid_constant__ CUtensorMap tmW, __nv_bfloat16* __restrict__ Q,
                         __nv_bfloat16* __restrict__ K, __nv_bfloat16* __restrict__ V, ProjDims p,
-                        int n_items, uint64_t wait_limit_ns) {
+                        int n_tiles, uint64_t wait_limit_ns) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -140,9 +116,8 @@ qkv_proj_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmX,
       int slot = 0;
       uint32_t phase = 0, issued = 0, issued_phase = 0;
       bool ok = true;
-      for (int t = blockIdx.x; ok && t < n_items; t += gridDim.x) {
-        const ProjItem w = proj_item(p, t);
-        const int m0 = w.m0, c0 = w.c0, npanels = w.width / 64;
+      for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x) {
+        const int m0 = (t / p.n_ntiles) * kBM, c0 = (t % p.n_ntiles) * kBN;
         for (int kt = 0; kt < p.n_ktiles; ++kt) {
           if (!wait_bounded(empty_bar(slot), phase ^ 1u, wc)) {
             ok = false;
@@ -151,11 +126,12 @@ qkv_proj_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmX,
           issued |= 1u << slot;
           issued_phase = (issued_phase & ~(1u << slot)) | (phase << slot);
           const uint32_t st = sbase + slot * kStageBytes;
-          mbar_arrive_expect_tx(full_bar(slot), kXBytes + npanels * kWPanelBytes);
-          // X: columns [kt*64, +64) of rows [m0, +128); W: rows [kt*64, +64), columns
-          // [c0, +width) as 64-column panels (rows past M or d and columns past ncol read as 0)
+          mbar_arrive_expect_tx(full_bar(slot), kStageBytes);
+          // X: columns [kt*64, +64) of rows [m0, +128); W: rows [kt*64, +64), columns [c0, +256)
+          // as four 64-column panels (rows past M or d and columns past ncol read as 0)
           tma_load_3d(st, &tmX, full_bar(slot), kt * kBK, m0, 0);
-          for (int q = 0; q < npanels; ++q)
+#pragma unroll
+          for (int q = 0; q < kBN / 64; ++q)
             tma_load_3d(st + kXBytes + q * kWPanelBytes, &tmW, full_bar(slot), c0 + 64 * q,
                         kt * kBK, 0);
           if (++slot == kStages) {
@@ -171,16 +147,16 @@ qkv_proj_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmX,
     }
   } else if (warp == kMmaWarp) {
     if (lane == 0) {
-      // C (+)= X W: M = 128 tokens, N = the item's width (256, 128 or 64 columns), K = 16 per
-      // MMA.  A = X tile K-major (32 B per step inside the 128-byte panel).  B = W tile MN-major:
-      // groups of 8 rows 1024 B apart (stride byte offset), 64-column panels kWPanelBytes apart
-      // (leading byte offset), 16 rows = 2048 B per step.
+      // C (+)= X W: M = 128 tokens, N = 256 columns, K = 16 per MMA.  A = X tile K-major (32 B
+      // per step inside the 128-byte panel).  B = W tile MN-major: groups of 8 rows 1024 B
+      // apart (stride byte offset), 64-column panels kWPanelBytes apart (leading byte offset),
+      // 16 rows = 2048 B per step.
+      constexpr uint32_t kIdesc = make_idesc(kBM, kBN, true);
       int slot = 0;
       uint32_t phase = 0;
       bool ok = true;
       int it = 0;
-      for (int t = blockIdx.x; ok && t < n_items; t += gridDim.x, ++it) {
-        const uint32_t idesc = make_idesc(kBM, proj_item(p, t).width, true);
+      for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x, ++it) {
         const int a = it & 1;
         const uint32_t tacc = tmem + a * kBN;
         // the epilogue has drained this accumulator (its use before last)
@@ -195,7 +171,7 @@ qkv_proj_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmX,
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk)
             mma_f16_ss(tacc, make_sdesc_sw128(st + kk * 32, 16, 1024),
-                       make_sdesc_sw128(st + kXBytes + kk * 2048, kWPanelBytes, 1024), idesc,
+                       make_sdesc_sw128(st + kXBytes + kk * 2048, kWPanelBytes, 1024), kIdesc,
                        (kt > 0 || kk > 0) ? 1u : 0u);
           mma_commit(empty_bar(slot));
           if (++slot == kStages) {
@@ -213,16 +189,15 @@ qkv_proj_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmX,
     const int r = lane_base + lane;
     const int hq = p.H * p.dk;
     int it = 0;
-    for (int t = blockIdx.x; t < n_items; t += gridDim.x, ++it) {
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
       const int a = it & 1;
       if (!wait_bounded(acc_full(a), uint32_t(it >> 1) & 1u, wc)) break;
       tc_fence_after_sync();
-      const ProjItem w = proj_item(p, t);
-      const int m = w.m0 + r, c0 = w.c0;
+      const int m = (t / p.n_ntiles) * kBM + r, c0 = (t % p.n_ntiles) * kBN;
       const bool row_ok = m < p.M;
       const int b = row_ok ? m / p.N : 0, n = row_ok ? m % p.N : 0;
 #pragma unroll 2
-      for (int c = 0; c < w.width; c += 32) {
+      for (int c = 0; c < kBN; c += 32) {
         uint32_t o[32];
         tmem_ld_32x32b_x32(tmem + (uint32_t(lane_base) << 16) + a * kBN + c, o);
         tmem_wait_ld();
@@ -502,8 +477,6 @@ int launch_qkv_proj_bf16(const ProjArgs& a, char* msg, size_t msglen) {
       return 5;
     }
     const int64_t clusters = n_pair_items < max_clusters ? n_pair_items : max_clusters;
-    p.n_full = 0;
-    p.pieces = 1;
     qkv_proj_bf16_mc_kernel<<<dim3(unsigned(2 * clusters)), dim3(kThreads), kSmemBytes,
                               a.stream>>>(mx, mw, static_cast<__nv_bfloat16*>(a.Q),
                                           static_cast<__nv_bfloat16*>(a.K),
@@ -517,23 +490,13 @@ int launch_qkv_proj_bf16(const ProjArgs& a, char* msg, size_t msglen) {
     return 0;
   }
   const int grid = int(n_tiles < sm_count ? n_tiles : sm_count);
-  // When the last round of CTAs is at most a quarter full, its tiles are cut into up to 4
-  // narrower items that still fit one round (measured: 4x2048x1024 -> 3072 has 8 such tiles on
-  // 152 SMs, +2.4 %; a round 42 % full gained nothing, its tiles already running faster with
-  // fewer CTAs sharing the L2).
-  const int64_t tail = n_tiles % grid;
-  int pieces = 1;
-  if (tail > 0 && 4 * tail <= grid) pieces = 4;
-  p.n_full = int(n_tiles - (pieces > 1 ? tail : 0));
-  p.pieces = pieces;
-  const int64_t n_items = p.n_full + (n_tiles - p.n_full) * pieces;
-  if (n_items > 0x7fffffffLL) {
+  if (n_tiles > 0x7fffffffLL) {
     snprintf(msg, msglen, "projection: too many tiles");
     return 3;
   }
   qkv_proj_bf16_tc_kernel<<<dim3(unsigned(grid)), dim3(kThreads), kSmemBytes, a.stream>>>(
       mx, mw, static_cast<__nv_bfloat16*>(a.Q), static_cast<__nv_bfloat16*>(a.K),
-      static_cast<__nv_bfloat16*>(a.V), p, int(n_items), wait_limit_ns());
+      static_cast<__nv_bfloat16*>(a.V), p, int(n_tiles), wait_limit_ns());
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     snprintf(msg, msglen, "projection launch: %s", cudaGetErrorString(e));

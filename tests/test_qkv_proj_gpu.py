@@ -106,9 +106,8 @@ def test_qkv_proj_feeds_attention(oracle):
 def test_qkv_proj_large_grids(oracle, shape):
     """Grids of several tiles per persistent CTA (both accumulators reused many times), checked
     on the first and the last 300 tokens of every batch entry (each token's outputs depend on
-    that token's row of X only).  The last tokens are the tiles of the last round, which are
-    cut into narrower pieces when they do not fill the GPU (768 tiles on 152 SMs: 8 tiles in
-    four 64-column pieces each)."""
+    that token's row of X only).  The last tokens come from the last, partly filled round of
+    the persistent clusters (both CTAs of a cluster, second of a pair of token blocks)."""
     B, N, d, H, dk, dv = shape
     r = np.random.default_rng(sum(shape))
     xf = r.normal(size=(B, N, d))
