@@ -136,3 +136,19 @@ def test_fused_rejects_other_shapes_and_dtypes():
     with pytest.raises(pkg.MoaError) as e:
         pkg.attn_bwd(q, k, v, o, lse, bf16_dev(gb), x.scale, fused=True)
     assert e.value.status == _lib.MOA_ERR_UNSUPPORTED_SHAPE
+
+
+def test_fused_bench_workload_sampled_heads(oracle):
+    """The fused backward on bench.py's default backward workload (bf16 B=4 H=16 N=2048 d=64,
+    the launch configuration `bench.py --pass bwd` times): three whole (b, h) slices, the last
+    one from the last CTAs of the grid, element by element against the oracle."""
+    cfg = I.CONFIGS[2]
+    x = I.make_inputs(cfg)
+    g, gb = I.make_grad_output(cfg)
+    dq, dk, dv = (t.float().cpu().numpy() for t in grads(x, gb, True))
+    for (b, h) in [(0, 0), (2, 7), (3, 15)]:
+        ref = oracle.attn_bwd(x.q[b:b + 1, h:h + 1], x.k[b:b + 1, h:h + 1], x.v[b:b + 1, h:h + 1],
+                              g[b:b + 1, h:h + 1], x.scale)
+        for name, a, r in zip(("dQ", "dK", "dV"), (dq, dk, dv), ref):
+            err = rel_err(a[b:b + 1, h:h + 1], r)
+            assert err <= BF16_TOL, f"workload 2 slice ({b},{h}) {name}: {err:.3e}"

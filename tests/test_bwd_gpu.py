@@ -159,3 +159,17 @@ def test_bwd_bench_workload_sampled_heads(oracle):
                               g[b:b + 1, h:h + 1], x.scale)
         got = tuple(t[b:b + 1, h:h + 1] for t in (dq, dk, dv))
         check_grads(got, ref, f"workload 2 slice ({b},{h})")
+
+
+def test_bwd_d128_workload_sampled_head(oracle):
+    """The three-kernel backward on the d=128 workload bench.py --pass bwd --workload 3 times
+    (bf16 B=2 H=32 N=8192), the last (b, h) slice against the oracle element by element."""
+    cfg = I.CONFIGS[3]
+    x = I.make_inputs(cfg)
+    g, gb = I.make_grad_output(cfg)
+    dq, dk, dv = run_bwd(x, gb)
+    b, h = 1, 31
+    ref = oracle.attn_bwd(x.q[b:b + 1, h:h + 1], x.k[b:b + 1, h:h + 1], x.v[b:b + 1, h:h + 1],
+                          g[b:b + 1, h:h + 1], x.scale)
+    got = tuple(t[b:b + 1, h:h + 1] for t in (dq, dk, dv))
+    check_grads(got, ref, f"workload 3 slice ({b},{h})")
