@@ -121,3 +121,20 @@ def test_qkv_proj_large_grids(oracle, shape):
             assert err <= 1e-2, f"{shape} {name} tokens {sl}: {err:.3e}"
     for a in got:
         assert np.all(np.isfinite(a))
+
+
+@pytest.mark.parametrize("shape", [(4, 2048, 1024, 16, 64, 64), (2, 8192, 4096, 32, 128, 128)],
+                         ids=["bench-workload-2", "bench-workload-3"])
+def test_qkv_proj_bench_shapes(oracle, shape):
+    """The projections bench.py --pass qkv times (the cluster kernel, every pair item of the
+    persistent grid), checked on the first and last 64 tokens of every batch entry."""
+    B, N, d, H, dk, dv = shape
+    r = np.random.default_rng(sum(shape))
+    xf = r.normal(size=(B, N, d))
+    wf = r.normal(size=(d, 2 * H * dk + H * dv)) / np.sqrt(d)
+    x32, w32, got = run(xf, wf, H, dk, dv)
+    for sl in (slice(0, 64), slice(N - 64, N)):
+        ref = oracle.qkv_proj(np.ascontiguousarray(x32[:, sl]), w32, H, dk, dv)
+        for name, a, b in zip("QKV", got, ref):
+            err = rel_err(a[:, :, sl], b)
+            assert err <= 1e-2, f"{shape} {name} tokens {sl}: {err:.3e}"
