@@ -1096,16 +1096,23 @@ attn_bwd_fused_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_cons
       ok = wait_bounded(dp_full, par, wc);
       if (!ok) break;
       tc_fence_after_sync();
-      tmem_load_part<kCols>(tDP, r);
+      // dP^T in two 16-column halves: all 32 columns beside P in registers spill at the
+      // 96-register cap of 19 warps.
 #pragma unroll
-      for (int q = 0; q < kCols; q += 4) {
-        const float4 d = d4[q >> 2];
-        const float s0 = p[q] * (__uint_as_float(r[q]) - d.x);
-        const float s1 = p[q + 1] * (__uint_as_float(r[q + 1]) - d.y);
-        const float s2 = p[q + 2] * (__uint_as_float(r[q + 2]) - d.z);
-        const float s3 = p[q + 3] * (__uint_as_float(r[q + 3]) - d.w);
-        pk[q >> 1] = pack_bf16x2(s0, s1);
-        pk[(q >> 1) + 1] = pack_bf16x2(s2, s3);
+      for (int h = 0; h < kCols; h += 16) {
+        tmem_ld_32x32b_x16(tDP + h, r);
+        tmem_wait_ld();
+        reg_anchor_x16(r);
+#pragma unroll
+        for (int q = 0; q < 16; q += 4) {
+          const float4 d = d4[(h + q) >> 2];
+          const float s0 = p[h + q] * (__uint_as_float(r[q]) - d.x);
+          const float s1 = p[h + q + 1] * (__uint_as_float(r[q + 1]) - d.y);
+          const float s2 = p[h + q + 2] * (__uint_as_float(r[q + 2]) - d.z);
+          const float s3 = p[h + q + 3] * (__uint_as_float(r[q + 3]) - d.w);
+          pk[(h + q) >> 1] = pack_bf16x2(s0, s1);
+          pk[((h + q) >> 1) + 1] = pack_bf16x2(s2, s3);
+        }
       }
       // dS(i) overwrites dS(i-1) once dK(i-1) and dQ(i-1) have read it.
       if (i > 0) {
