@@ -19,18 +19,22 @@
 //     them directly.  V is the "MN-major" B operand, again as stored.
 //   * Step IV (division, Section 4.5) is applied once per row in the epilogue: O / l.
 //
-// CTA organisation (one CTA per SM: 512 TMEM columns, up to ~192 KB shared memory):
+// CTA organisation, two-tile kernel (one CTA per SM: 512 TMEM columns, up to ~192 KB shared
+// memory):
 //   work item = (b*H + h, block of 256 query rows) = two 128-row Q tiles;
 //   warps 0-3: softmax + epilogue of Q tile 0; warps 4-7: same for Q tile 1
 //              (thread t of such a warpgroup owns query row t of its tile);
 //   warp 8:    TMEM allocation; issues tcgen05.mma (both tiles, or tile 0 only, see below);
 //   warp 9:    the single thread that issues all TMA loads;
 //   warp 10:   issues tcgen05.mma for tile 1 when P has TMEM columns of its own.
+// One-tile kernel (d_k = d_v = 64 without a split key axis; two CTAs per SM, 256 TMEM columns
+// and ~98 KB of shared memory each): work item = (b*H + h, block of 128 query rows); warps 0-3
+// softmax + epilogue, warp 4 TMEM allocation and tcgen05.mma, warp 5 TMA loads.
 // K and V tiles of 128 keys stream through an NS-stage shared-memory ring.  Two schedules:
 //   d_v = 128 (TMEM: S0 S1 O0 O1): P_j is written over S_j's columns, so per key tile n >= 1
 //     the single issuing thread runs O_j += P_j(n-1) V(n-1) and then S_j = Q_j K(n)^T, tile 0
 //     then tile 1; ring order K0 V0 K1 V1 ...
-//   d_v = 64 (TMEM: S0 S1 P0 P1 O0 O1): P_j has columns of its own.  As soon as the softmax has
+//   d_v = 64 (TMEM: S0 S1 P0 P1 O0 O1, one tile: S0 P0 O0): P_j has columns of its own.  As soon as the softmax has
 //     read S_j(n) into registers, tile j's issuing thread computes S_j(n+1), and it runs
 //     O_j += P_j(n) V(n) once P_j(n) is written, so the softmax never waits for the product
 //     with V; ring order K0 K1 V0 K2 V1 ...
@@ -62,21 +66,28 @@ using namespace tc;
 
 constexpr int kBM = 128;          // query rows per Q tile (= TMEM lanes)
 constexpr int kBN = 128;          // keys per K/V tile
-constexpr int kQTiles = 2;        // Q tiles per CTA
-constexpr int kThreads = 352;     // 8 softmax warps, MMA warp (tile 0), TMA warp, MMA warp (tile 1)
-constexpr int kMmaWarp0 = 8;      // also allocates and frees TMEM
-constexpr int kLoadWarp = 9;
-constexpr int kMmaWarp1 = 10;
-constexpr int kTmemCols = 512;
+constexpr int kQTiles = 2;        // Q tiles per CTA of the two-tile kernel
 constexpr float kRescaleLog2 = 8.0f;  // lazy-rescale threshold: exponentials stay <= 2^8
-// Longest suspension of one mbarrier test for the d_v = 64 schedule, where the MMA and TMA
-// threads wait long enough that polling would take issue slots from the softmax warps
-// (measured +3.6% there, -1..3% with d_v = 128, which therefore polls).
+// Longest suspension of one mbarrier test for the two-tile d_v = 64 schedule, where the MMA
+// and TMA threads wait long enough that polling would take issue slots from the softmax warps
+// (measured +3.6% there, -1..3% with d_v = 128, which therefore polls).  One-tile CTAs poll:
+// with the suspension they ran at 709 TFLOP/s instead of 740 on 4x16x2048^2.
 constexpr uint32_t kWaitHintNs = 20000;
 
-template <int DK, int DV>
+template <int DK, int DV, int QT = 2>
 struct Cfg {
   static_assert(DK == 64 || DK == 128, "d_k must be 64 or 128");
+  static_assert(QT == 1 || QT == 2, "one or two Q tiles per CTA");
+  static_assert(QT == 2 || DV == 64, "one-tile CTAs use the separate-P schedule");
+  // Warps: 4 softmax warps per Q tile, then the MMA warp of tile 0 (it also allocates and frees
+  // TMEM), the TMA warp and, with two tiles, the MMA warp of tile 1.  One-tile CTAs run two per
+  // SM (half the registers, TMEM and shared memory each).
+  static constexpr int kThreads = QT == 2 ? 352 : 192;
+  static constexpr int kMinBlocks = QT == 2 ? 1 : 2;
+  static constexpr int kMmaWarp0 = 4 * QT;
+  static constexpr int kLoadWarp = 4 * QT + 1;
+  static constexpr int kMmaWarp1 = QT == 2 ? 10 : -1;
+  static constexpr int kTmemCols = 256 * QT;
   static_assert(DV == 64 || DV == 128, "d_v must be 64 or 128");
   // One 128-byte swizzle panel holds 64 bf16 columns of 128 rows: 16 KB.
   static constexpr int kPanelBytes = 128 * 128;
@@ -84,9 +95,9 @@ struct Cfg {
   static constexpr int kKTileBytes = kBN * DK * 2;
   static constexpr int kVTileBytes = kBN * DV * 2;
   static constexpr int kStageBytes = kKTileBytes > kVTileBytes ? kKTileBytes : kVTileBytes;
-  static constexpr int kStages = (DK == 64 && DV == 64) ? 8 : 4;
+  static constexpr int kStages = QT == 1 ? (DK == 64 ? 5 : 2) : (DK == 64 && DV == 64) ? 8 : 4;
   static constexpr int kOffQ = 0;
-  static constexpr int kOffKV = kOffQ + kQTiles * kQTileBytes;
+  static constexpr int kOffKV = kOffQ + QT * kQTileBytes;
   static constexpr int kOffBar = kOffKV + kStages * kStageBytes;
   // P in TMEM columns of its own (d_v = 64: S0 S1 P0 P1 O0 O1 fill the 512 columns) lets the
   // next block's scores be computed while the softmax still works on this block.  With
@@ -95,16 +106,19 @@ struct Cfg {
   // With separate P, each Q tile gets its own issuing thread (its chain of products never
   // waits behind the other tile's).  With P aliasing S, one thread issues both tiles' products
   // back to back, which lets the first tile's scores finish early.
-  static constexpr int kIssuers = kSepP ? 2 : 1;
+  static constexpr int kIssuers = kSepP ? QT : 1;
   // barriers: full[NS], empty[NS], q_full, s_full[2], p_ready[2], o_done[2], s_free[2], p_free[2]
   static constexpr int kNumBars = 2 * kStages + 11;
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
   static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack for 1024-B alignment
+  // Two tiles: S0 S1 P0 P1 O0 O1 (separate P) or S0 S1 O0 O1.  One tile: S0 P0 O0.
   static constexpr uint32_t kTmemS0 = 0, kTmemS1 = 128;
-  static constexpr uint32_t kTmemP0 = kSepP ? 256 : kTmemS0, kTmemP1 = kSepP ? 320 : kTmemS1;
-  static constexpr uint32_t kTmemO0 = kSepP ? 384 : 256, kTmemO1 = kTmemO0 + DV;
-  static_assert(kTmemO1 + DV <= kTmemCols, "TMEM budget");
-  static_assert(kSmemBytes <= 232448, "shared memory budget");
+  static constexpr uint32_t kTmemP0 = kSepP ? 128 * QT : kTmemS0;
+  static constexpr uint32_t kTmemP1 = kSepP ? 320 : kTmemS1;
+  static constexpr uint32_t kTmemO0 = kSepP ? 192 * QT : 256, kTmemO1 = kTmemO0 + DV;
+  static_assert((QT == 2 ? kTmemO1 : kTmemO0) + DV <= kTmemCols, "TMEM budget");
+  // Per SM: 228 KB, 1 KB of it reserved per CTA.
+  static_assert(kSmemBytes <= (QT == 2 ? 232448 : 233472 / 2 - 1024), "shared memory budget");
 };
 
 // Maximum of 128 values (of their negations if NEG) with four independent 3-input chains.
@@ -142,15 +156,19 @@ __device__ __forceinline__ void tmem_scale_row(uint32_t taddr, float alpha) {
 
 // SPLIT: this CTA covers one range of the key axis and writes fp32 partials for the merge kernel
 // (separate instantiation, so the unsplit kernel carries none of it).
-template <int DK, int DV, bool SPLIT>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int DK, int DV, bool SPLIT, int QT>
+__global__ void __launch_bounds__(Cfg<DK, DV, QT>::kThreads, Cfg<DK, DV, QT>::kMinBlocks)
 attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmK,
                         const __grid_constant__ CUtensorMap tmV, __nv_bfloat16* __restrict__ O,
                         int Nq, int Nk, int n_qblocks, float c_log2, uint64_t wait_limit_ns,
                         int n_splits, int kv_per_split, float* __restrict__ ws_o,
                         float2* __restrict__ ws_ml, float* __restrict__ lse) {
-  using C = Cfg<DK, DV>;
+  using C = Cfg<DK, DV, QT>;
+  static_assert(!SPLIT || QT == 2, "split key axes use two-tile CTAs");
+  constexpr int kQTiles = QT;
+  constexpr int kMmaWarp0 = C::kMmaWarp0, kLoadWarp = C::kLoadWarp, kMmaWarp1 = C::kMmaWarp1;
+  constexpr int kTmemCols = C::kTmemCols;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -175,7 +193,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  // CTA -> (b*H + h, 256-row query block, key split); splits of one block are adjacent, and
+  // CTA -> (b*H + h, 128·QT-row query block, key split); splits of one block are adjacent, and
   // blocks of one head are adjacent (head-major), so concurrently running CTAs share K/V in L2.
   const int split = SPLIT ? int(blockIdx.x % n_splits) : 0;
   const int item = SPLIT ? int(blockIdx.x / n_splits) : int(blockIdx.x);
@@ -184,7 +202,8 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   // This CTA's key blocks: [kb0, kb0 + n_kt) (all of them unless the key axis is split).
   const int kb0 = SPLIT ? split * kv_per_split : 0;
   const int n_kt = SPLIT ? min((Nk + kBN - 1) / kBN - kb0, kv_per_split) : (Nk + kBN - 1) / kBN;
-  const WaitCtl wc{abort_flag, wait_limit_ns, C::kSepP ? kWaitHintNs : 0u, &g_moa_bf16_status};
+  const WaitCtl wc{abort_flag, wait_limit_ns, C::kSepP && QT == 2 ? kWaitHintNs : 0u,
+                   &g_moa_bf16_status};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
@@ -613,7 +632,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   // Teardown: wait for the tensor core to go quiet before freeing TMEM.
   if (warp == kMmaWarp0) {
     wait_quiesce(o_done(0), 0, wait_limit_ns, &g_moa_bf16_status);
-    wait_quiesce(o_done(1), 0, wait_limit_ns, &g_moa_bf16_status);
+    if (QT == 2) wait_quiesce(o_done(1), 0, wait_limit_ns, &g_moa_bf16_status);
   }
   tc_fence_before_sync();
   __syncthreads();
@@ -750,30 +769,43 @@ bool encode_f32_map_sw128(CUtensorMap* map, const void* base, int64_t BH, int64_
 
 namespace {
 
+// One-tile CTAs, two per SM, for d_k = d_v = 64 when the key axis is not split: the two CTAs
+// on an SM can overlap each other's start-up and epilogue (measured 680 -> 740 TFLOP/s on
+// 4x16x2048^2; SM active cycles 81 % -> 91 %).  With d_k = 128 only two
+// 32 KB ring stages fit beside the Q tile, and the two-tile kernel stays faster (1063 vs 981).
+template <int DK, int DV>
+constexpr bool kUseOneTile = DV == 64 && DK == 64;
+
 template <int DK, int DV>
 int launch_tc(const AttnArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
               const CUtensorMap& mv, const SplitPlan& sp, void* ws, char* msg, size_t msglen) {
   using C = Cfg<DK, DV>;
+  constexpr int QT1 = kUseOneTile<DK, DV> ? 1 : 2;
+  using C1 = Cfg<DK, DV, QT1>;
   if (sp.n_splits > 1 && a.lse != nullptr) {
     snprintf(msg, msglen, "the log-sum-exp output is not available with a split key axis");
     return 1;
   }
-  auto kern = sp.n_splits > 1 ? attn_fwd_bf16_tc_kernel<DK, DV, true>
-                              : attn_fwd_bf16_tc_kernel<DK, DV, false>;
+  const bool split = sp.n_splits > 1;
+  auto kern = split ? attn_fwd_bf16_tc_kernel<DK, DV, true, 2>
+                    : attn_fwd_bf16_tc_kernel<DK, DV, false, QT1>;
+  const int threads = split ? C::kThreads : C1::kThreads;
+  const int smem_bytes = split ? C::kSmemBytes : C1::kSmemBytes;
+  const int tile_rows = split ? kQTiles * kBM : QT1 * kBM;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(attn_fwd_bf16_tc_kernel<DK, DV, false>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    attr_err = cudaFuncSetAttribute(attn_fwd_bf16_tc_kernel<DK, DV, false, QT1>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C1::kSmemBytes);
     if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(attn_fwd_bf16_tc_kernel<DK, DV, true>,
+      attr_err = cudaFuncSetAttribute(attn_fwd_bf16_tc_kernel<DK, DV, true, 2>,
                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   });
   if (attr_err != cudaSuccess) {
     snprintf(msg, msglen, "cudaFuncSetAttribute (bf16 kernel): %s", cudaGetErrorString(attr_err));
     return 5;
   }
-  const int64_t n_qblocks = (a.Nq + kQTiles * kBM - 1) / (kQTiles * kBM);
+  const int64_t n_qblocks = (a.Nq + tile_rows - 1) / tile_rows;
   const int64_t grid = a.B * a.H * n_qblocks * sp.n_splits;
   if (grid > 0x7fffffffLL) {
     snprintf(msg, msglen, "bf16 path: %lld CTAs exceeds the grid limit", (long long)grid);
@@ -785,7 +817,7 @@ int launch_tc(const AttnArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
   float2* ws_ml = sp.n_splits > 1
                       ? reinterpret_cast<float2*>(static_cast<float*>(ws) + sp.n_splits * rows * DV)
                       : nullptr;
-  kern<<<dim3(unsigned(grid)), dim3(kThreads), C::kSmemBytes, a.stream>>>(
+  kern<<<dim3(unsigned(grid)), dim3(threads), smem_bytes, a.stream>>>(
       mq, mk, mv, static_cast<__nv_bfloat16*>(a.O), int(a.Nq), int(a.Nk), int(n_qblocks), c_log2,
       wait_limit_ns(), sp.n_splits, sp.kv_per_split, ws_o, ws_ml, a.lse);
   cudaError_t e = cudaGetLastError();
