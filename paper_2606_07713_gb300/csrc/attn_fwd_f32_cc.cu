@@ -16,13 +16,15 @@
 // Two kernels:
 //   attn_fwd_f32_cc_kernel   CTA of 128 threads = 4 warps, BM = 32 rows (8 per warp), BN = 64
 //                            keys; K and V tiles shared by the CTA's 32 rows through smem.
-//   attn_fwd_f32_row_kernel  one warp per query row (lane = key of a 32-key chunk for the
-//                            scores, lane = output column for the sum over V), for problems too
-//                            small to give every SM a 32-row CTA: the work spreads over up to
-//                            32x as many warps, which matters when the call is latency-bound.
+//   attn_fwd_f32_small_kernel  8 query rows of one (b, h) per CTA, one warp per row, for
+//                            problems too small to give every SM a 32-row CTA: 64-key chunks of
+//                            K and V are copied with cp.async, every piece of a chunk in flight
+//                            at once, double-buffered, which matters when the call is bound by
+//                            memory latency.
 #include <cuda_runtime.h>
 #include <math.h>
 #include <cstdio>
+#include <mutex>
 
 #include "internal.h"
 
@@ -173,117 +175,201 @@ attn_fwd_f32_cc_kernel(const float* __restrict__ Q, const float* __restrict__ K,
   }
 }
 
-// One warp per query row r = (b*H + h)*N_q + i; 8 rows per CTA.
-__global__ void __launch_bounds__(256)
-attn_fwd_f32_row_kernel(const float* __restrict__ Q, const float* __restrict__ K,
-                        const float* __restrict__ V, float* __restrict__ O,
-                        float* __restrict__ lse, int Nq, int Nk, int dk, int dv, float scale,
-                        long long rows) {
-  __shared__ float sq[8][kMaxD];
+// Small problems: 8 query rows of one (b, h) per CTA, one warp per row.  The CTA's 256
+// threads copy 64-key chunks of K and V into shared memory with cp.async (16-byte pieces, all
+// in flight at once), double-buffered: chunk c+1 is requested before chunk c is used, so a call
+// that is bound by memory latency pays it about once per chunk pair instead of once per
+// dependent load.  Per chunk, lane = key for the scores (keys lane and lane + 32), lane =
+// output column for the sum over V.
+constexpr int kSmallRows = 8;     // rows (= warps) per CTA
+constexpr int kSmallKeys = 64;    // keys per chunk
+constexpr int kSmallThreads = 32 * kSmallRows;
+
+struct SmallSmem {
+  // K rows padded by 4 floats: 16-byte aligned, and the float4 reads of 8 consecutive key rows
+  // fall on disjoint banks.
+  __host__ __device__ static int ldk(int dk) { return dk + 4; }
+  static size_t bytes(int dk, int dv) {
+    return sizeof(float) * (size_t(kSmallRows) * dk + 2 * size_t(kSmallKeys) * ldk(dk) +
+                            2 * size_t(kSmallKeys) * dv + size_t(kSmallRows) * kSmallKeys);
+  }
+};
+
+// 16 bytes global -> shared, asynchronous; src_bytes = 0 writes zeros (the source is not read).
+__device__ __forceinline__ void cp_async16(float* dst, const float* src, int src_bytes) {
+  const unsigned d = static_cast<unsigned>(__cvta_generic_to_shared(dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+__global__ void __launch_bounds__(kSmallThreads)
+attn_fwd_f32_small_kernel(const float* __restrict__ Q, const float* __restrict__ K,
+                          const float* __restrict__ V, float* __restrict__ O,
+                          float* __restrict__ lse, int Nq, int Nk, int dk, int dv, int n_qtiles,
+                          float scale) {
+  extern __shared__ __align__(16) float smem[];
+  const int ldk = SmallSmem::ldk(dk);
+  float* sQ = smem;                                   // [8][dk]
+  float* sK = sQ + kSmallRows * dk;                   // [2][64][dk + 4]
+  float* sV = sK + 2 * kSmallKeys * ldk;              // [2][64][dv]
+  float* sP = sV + 2 * kSmallKeys * dv;               // [8][64]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long r = (long long)blockIdx.x * 8 + warp;
-  if (r >= rows) return;  // whole warps leave together
-  const long long bh = r / Nq;
-  const float* q = Q + r * dk;
+  const long long bh = blockIdx.x / n_qtiles;
+  const int row = (blockIdx.x % n_qtiles) * kSmallRows + warp;  // query row of this warp
+  const bool active = row < Nq;
   const float* Kh = K + bh * (long long)Nk * dk;
   const float* Vh = V + bh * (long long)Nk * dv;
-  for (int j = lane; j < dk; j += 32) sq[warp][j] = q[j];
-  __syncwarp();
+
+  const int kseg = dk / 4, vseg = dv / 4;  // 16-byte pieces per row (d is a multiple of 4)
+  auto request = [&](int c) {             // chunk c -> buffer c % 2
+    const int k0 = c * kSmallKeys, b = c & 1;
+    float* dK = sK + b * kSmallKeys * ldk;
+    float* dV = sV + b * kSmallKeys * dv;
+    for (int i = threadIdx.x; i < kSmallKeys * kseg; i += kSmallThreads) {
+      const int r = i / kseg, j = i - r * kseg;
+      const bool in = k0 + r < Nk;
+      cp_async16(dK + r * ldk + 4 * j, in ? Kh + (long long)(k0 + r) * dk + 4 * j : Kh, in ? 16 : 0);
+    }
+    for (int i = threadIdx.x; i < kSmallKeys * vseg; i += kSmallThreads) {
+      const int r = i / vseg, j = i - r * vseg;
+      const bool in = k0 + r < Nk;
+      cp_async16(dV + r * dv + 4 * j, in ? Vh + (long long)(k0 + r) * dv + 4 * j : Vh, in ? 16 : 0);
+    }
+    cp_async_commit();
+  };
+
+  request(0);
+  if (active)
+    for (int j = lane; j < dk; j += 32) sQ[warp * dk + j] = Q[(bh * Nq + row) * (long long)dk + j];
+  const float* q = sQ + warp * dk;
+  float* p_row = sP + warp * kSmallKeys;
+
   float m = -INFINITY, l = 0.f;
   float acc[kMaxColGroups];
 #pragma unroll
   for (int g = 0; g < kMaxColGroups; ++g) acc[g] = 0.f;
-  for (int k0 = 0; k0 < Nk; k0 += 32) {
-    // lane = key k0 + lane: its score (rows past N_k: -inf)
-    const int key = k0 + lane;
-    float s = -INFINITY;
-    if (key < Nk) {
-      const float* kr = Kh + (long long)key * dk;
-      float d = 0.f;
-      // groups of 4 float4 loads in flight before their products
-      for (int j0 = 0; j0 < dk; j0 += 16) {
-        float4 kv[4];
+  const int n_chunks = (Nk + kSmallKeys - 1) / kSmallKeys;
+  for (int c = 0; c < n_chunks; ++c) {
+    if (c + 1 < n_chunks) {
+      request(c + 1);  // its buffer was released by the barrier at the end of chunk c - 1
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();  // chunk c (and the Q rows) visible to every warp
+    if (active) {
+      const int k0 = c * kSmallKeys, b = c & 1;
+      const float* cK = sK + b * kSmallKeys * ldk;
+      const float* cV = sV + b * kSmallKeys * dv;
+      // scores of keys k0 + lane and k0 + lane + 32
+      const float* ka = cK + lane * ldk;
+      const float* kb = cK + (lane + 32) * ldk;
+      float s0 = 0.f, s1 = 0.f;
+      for (int j = 0; j < dk; j += 4) {
+        const float4 qv = *reinterpret_cast<const float4*>(q + j);
+        const float4 a4 = *reinterpret_cast<const float4*>(ka + j);
+        const float4 b4 = *reinterpret_cast<const float4*>(kb + j);
+        s0 = fmaf(qv.x, a4.x, s0);
+        s1 = fmaf(qv.x, b4.x, s1);
+        s0 = fmaf(qv.y, a4.y, s0);
+        s1 = fmaf(qv.y, b4.y, s1);
+        s0 = fmaf(qv.z, a4.z, s0);
+        s1 = fmaf(qv.z, b4.z, s1);
+        s0 = fmaf(qv.w, a4.w, s0);
+        s1 = fmaf(qv.w, b4.w, s1);
+      }
+      const float x0 = k0 + lane < Nk ? s0 * scale : -INFINITY;
+      const float x1 = k0 + lane + 32 < Nk ? s1 * scale : -INFINITY;
+      float cmax = fmaxf(x0, x1);
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
-          kv[u] = j0 + 4 * u < dk ? *reinterpret_cast<const float4*>(kr + j0 + 4 * u)
-                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int off = 16; off > 0; off >>= 1) cmax = fmaxf(cmax, __shfl_xor_sync(0xffffffffu, cmax, off));
+      const float mnew = fmaxf(m, cmax);  // finite: every chunk has at least one key
+      const float alpha = expf(m - mnew);  // exp(-inf) = 0 on the first chunk
+      const float p0 = expf(x0 - mnew), p1 = expf(x1 - mnew);
+      float psum = p0 + p1;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) psum += __shfl_xor_sync(0xffffffffu, psum, off);
+      l = l * alpha + psum;
+      m = mnew;
+      p_row[lane] = p0;
+      p_row[lane + 32] = p1;
+      __syncwarp();
+      // lane = output column: acc = alpha * acc + sum over the chunk's keys of p_k V[k, c]
+#pragma unroll
+      for (int g = 0; g < kMaxColGroups; ++g) acc[g] *= alpha;
+      const int kn = min(kSmallKeys, Nk - k0);
+      for (int k = 0; k < kn; k += 4) {
+        float pv[4], vv[4][kMaxColGroups];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          const int j = j0 + 4 * u;
-          if (j < dk) {
-            d = fmaf(sq[warp][j], kv[u].x, d);
-            d = fmaf(sq[warp][j + 1], kv[u].y, d);
-            d = fmaf(sq[warp][j + 2], kv[u].z, d);
-            d = fmaf(sq[warp][j + 3], kv[u].w, d);
+          pv[u] = k + u < kn ? p_row[k + u] : 0.f;  // zero-filled rows past N_k also read 0
+#pragma unroll
+          for (int g = 0; g < kMaxColGroups; ++g) {
+            const int col = lane + 32 * g;
+            vv[u][g] = col < dv ? cV[(k + u) * dv + col] : 0.f;
           }
         }
-      }
-      s = d * scale;
-    }
-    float cmax = s;
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) cmax = fmaxf(cmax, __shfl_xor_sync(0xffffffffu, cmax, off));
-    const float mnew = fmaxf(m, cmax);       // finite: every chunk has at least one key
-    const float alpha = expf(m - mnew);      // exp(-inf) = 0 on the first chunk
-    const float p = expf(s - mnew);          // 0 for keys past N_k
-    float psum = p;
+        for (int u = 0; u < 4; ++u)
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) psum += __shfl_xor_sync(0xffffffffu, psum, off);
-    l = l * alpha + psum;
-    m = mnew;
-    // lane = output column: acc = alpha * acc + sum over the chunk's keys of p_k V[k, c]
-    const int kn = min(32, Nk - k0);
-#pragma unroll
-    for (int g = 0; g < kMaxColGroups; ++g) acc[g] *= alpha;
-    // eight value rows loaded before their products (keys past N_k read as 0 with p = 0)
-    for (int kb = 0; kb < kn; kb += 8) {
-      float vv[8][kMaxColGroups];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const float* vr = Vh + (long long)(k0 + kb + u) * dv;
-#pragma unroll
-        for (int g = 0; g < kMaxColGroups; ++g) {
-          const int c = lane + 32 * g;
-          vv[u][g] = (kb + u < kn && c < dv) ? vr[c] : 0.f;
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const float pk = __shfl_sync(0xffffffffu, p, (kb + u) & 31);
-#pragma unroll
-        for (int g = 0; g < kMaxColGroups; ++g) acc[g] = fmaf(pk, vv[u][g], acc[g]);
+          for (int g = 0; g < kMaxColGroups; ++g) acc[g] = fmaf(pv[u], vv[u][g], acc[g]);
       }
     }
+    __syncthreads();  // buffer c % 2 and the P rows are free again
   }
-  const float inv = 1.0f / l;
+  if (active) {
+    const float inv = 1.0f / l;
+    float* orow = O + (bh * Nq + row) * (long long)dv;
 #pragma unroll
-  for (int g = 0; g < kMaxColGroups; ++g) {
-    const int c = lane + 32 * g;
-    if (c < dv) O[r * dv + c] = acc[g] * inv;
+    for (int g = 0; g < kMaxColGroups; ++g) {
+      const int col = lane + 32 * g;
+      if (col < dv) orow[col] = acc[g] * inv;
+    }
+    // ln sum_k exp(scale s_k) = m + ln l (m is the exact row maximum here)
+    if (lse != nullptr && lane == 0) lse[bh * Nq + row] = m + logf(l);
   }
-  if (lse != nullptr && lane == 0) lse[r] = m + logf(l);
 }
 
 }  // namespace
 
 int launch_attn_fwd_f32(const AttnArgs& a, char* msg, size_t msglen) {
-  // Few 32-row CTAs (fewer than two per SM): one warp per row instead.
+  // Few 32-row CTAs (fewer than two per SM): 8-row CTAs instead, each with its K/V chunks
+  // requested all at once.
   int dev = 0, sms = 148;
   if (cudaGetDevice(&dev) == cudaSuccess)
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const long long rows = (long long)a.B * a.H * a.Nq;
   if ((long long)a.B * a.H * ((a.Nq + kBM - 1) / kBM) < 2LL * sms) {
-    if ((rows + 7) / 8 > 0x7fffffffLL) {
+    const int n_qtiles = int((a.Nq + kSmallRows - 1) / kSmallRows);
+    const long long grid = (long long)a.B * a.H * n_qtiles;
+    if (grid > 0x7fffffffLL) {
       snprintf(msg, msglen, "fp32 path: too many rows");
       return 3;
     }
-    attn_fwd_f32_row_kernel<<<dim3(unsigned((rows + 7) / 8)), dim3(256), 0, a.stream>>>(
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [] {
+      attr_err = cudaFuncSetAttribute(attn_fwd_f32_small_kernel,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      int(SmallSmem::bytes(kMaxD, kMaxD)));
+    });
+    if (attr_err != cudaSuccess) {
+      snprintf(msg, msglen, "cudaFuncSetAttribute (fp32 small kernel): %s",
+               cudaGetErrorString(attr_err));
+      return 5;
+    }
+    attn_fwd_f32_small_kernel<<<dim3(unsigned(grid)), dim3(kSmallThreads),
+                                SmallSmem::bytes(int(a.dk), int(a.dv)), a.stream>>>(
         static_cast<const float*>(a.Q), static_cast<const float*>(a.K),
         static_cast<const float*>(a.V), static_cast<float*>(a.O), a.lse, int(a.Nq), int(a.Nk),
-        int(a.dk), int(a.dv), a.scale, rows);
+        int(a.dk), int(a.dv), n_qtiles, a.scale);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) {
-      snprintf(msg, msglen, "fp32 row kernel launch: %s", cudaGetErrorString(e));
+      snprintf(msg, msglen, "fp32 small kernel launch: %s", cudaGetErrorString(e));
       return 5;
     }
     return 0;
