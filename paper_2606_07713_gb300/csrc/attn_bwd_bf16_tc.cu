@@ -39,7 +39,6 @@
 
 #include <cmath>
 #include <cstdio>
-#include <mutex>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -1191,15 +1190,11 @@ int launch_bwd(const BwdArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
                const CUtensorMap& mv, const CUtensorMap& mdo, char* msg, size_t msglen) {
   using A = DkDvCfg<DK, DV>;
   using B = DqCfg<DK, DV>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(attn_bwd_dkdv_kernel<DK, DV>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, A::kSmemBytes);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(attn_bwd_dq_kernel<DK, DV>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, B::kSmemBytes);
-  });
+  cudaError_t attr_err =
+      ensure_smem_limit(reinterpret_cast<const void*>(attn_bwd_dkdv_kernel<DK, DV>), A::kSmemBytes);
+  if (attr_err == cudaSuccess)
+    attr_err =
+        ensure_smem_limit(reinterpret_cast<const void*>(attn_bwd_dq_kernel<DK, DV>), B::kSmemBytes);
   if (attr_err != cudaSuccess) {
     snprintf(msg, msglen, "cudaFuncSetAttribute (bf16 backward): %s", cudaGetErrorString(attr_err));
     return 5;
@@ -1249,12 +1244,8 @@ template <int DK, int DV>
 int launch_bwd_fused(const BwdArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
                      const CUtensorMap& mv, const CUtensorMap& mdo, char* msg, size_t msglen) {
   using F = FusedCfg<DK, DV>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(attn_bwd_fused_kernel<DK, DV>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, F::kSmemBytes);
-  });
+  const cudaError_t attr_err =
+      ensure_smem_limit(reinterpret_cast<const void*>(attn_bwd_fused_kernel<DK, DV>), F::kSmemBytes);
   if (attr_err != cudaSuccess) {
     snprintf(msg, msglen, "cudaFuncSetAttribute (fused backward): %s", cudaGetErrorString(attr_err));
     return 5;

@@ -292,11 +292,9 @@ int launch_attn_bwd_f32(const BwdArgs& a, char* msg, size_t msglen) {
                                          size_t(kChunk) * (dk + 1) + size_t(kChunk) * (dv + 1) +
                                          size_t(kWarps) * kRowsPerWarp * kChunk);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_bwd_f32_dkdv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             int(smem_kv));
+    e = ensure_smem_limit(reinterpret_cast<const void*>(attn_bwd_f32_dkdv_kernel), int(smem_kv));
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_bwd_f32_dq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             int(smem_q));
+    e = ensure_smem_limit(reinterpret_cast<const void*>(attn_bwd_f32_dq_kernel), int(smem_q));
   if (e == cudaSuccess) {
     attn_bwd_f32_dkdv_kernel<<<dim3(unsigned(BH * n_kt)), dim3(kThreads), smem_kv, a.stream>>>(
         static_cast<const float*>(a.Q), static_cast<const float*>(a.K),

@@ -792,15 +792,7 @@ int launch_tc(const AttnArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
   const int threads = split ? C::kThreads : C1::kThreads;
   const int smem_bytes = split ? C::kSmemBytes : C1::kSmemBytes;
   const int tile_rows = split ? kQTiles * kBM : QT1 * kBM;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(attn_fwd_bf16_tc_kernel<DK, DV, false, QT1>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C1::kSmemBytes);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(attn_fwd_bf16_tc_kernel<DK, DV, true, 2>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
-  });
+  const cudaError_t attr_err = ensure_smem_limit(reinterpret_cast<const void*>(kern), smem_bytes);
   if (attr_err != cudaSuccess) {
     snprintf(msg, msglen, "cudaFuncSetAttribute (bf16 kernel): %s", cudaGetErrorString(attr_err));
     return 5;

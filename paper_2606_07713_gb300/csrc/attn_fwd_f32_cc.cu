@@ -24,7 +24,6 @@
 #include <cuda_runtime.h>
 #include <math.h>
 #include <cstdio>
-#include <mutex>
 
 #include "internal.h"
 
@@ -350,13 +349,9 @@ int launch_attn_fwd_f32(const AttnArgs& a, char* msg, size_t msglen) {
       snprintf(msg, msglen, "fp32 path: too many rows");
       return 3;
     }
-    static std::once_flag once;
-    static cudaError_t attr_err = cudaSuccess;
-    std::call_once(once, [] {
-      attr_err = cudaFuncSetAttribute(attn_fwd_f32_small_kernel,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      int(SmallSmem::bytes(kMaxD, kMaxD)));
-    });
+    const cudaError_t attr_err =
+        ensure_smem_limit(reinterpret_cast<const void*>(attn_fwd_f32_small_kernel),
+                          int(SmallSmem::bytes(kMaxD, kMaxD)));
     if (attr_err != cudaSuccess) {
       snprintf(msg, msglen, "cudaFuncSetAttribute (fp32 small kernel): %s",
                cudaGetErrorString(attr_err));
@@ -381,8 +376,7 @@ int launch_attn_fwd_f32(const AttnArgs& a, char* msg, size_t msglen) {
     return 3;
   }
   const size_t smem = F32Smem::bytes(int(a.dk), int(a.dv));
-  cudaError_t e = cudaFuncSetAttribute(attn_fwd_f32_cc_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  cudaError_t e = ensure_smem_limit(reinterpret_cast<const void*>(attn_fwd_f32_cc_kernel), int(smem));
   if (e != cudaSuccess) {
     snprintf(msg, msglen, "cudaFuncSetAttribute (fp32 kernel): %s", cudaGetErrorString(e));
     return 5;

@@ -44,6 +44,10 @@ size_t splitkv_workspace_bytes(int64_t rows, int64_t dv, const SplitPlan& sp);
 // SM count of the current device, asked once per device.
 cudaError_t device_sm_count(int* sms);
 
+// Raises `func`'s dynamic shared-memory limit to `bytes` on the current device.  The attribute is
+// per device, so the call is made once per (kernel, device, size) and its result remembered.
+cudaError_t ensure_smem_limit(const void* func, int bytes);
+
 // Size of the fixed device array behind the allocation-free split entry point (16 MiB).
 constexpr size_t kNoallocScratchBytes = size_t(16) << 20;
 

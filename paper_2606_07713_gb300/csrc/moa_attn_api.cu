@@ -9,6 +9,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <vector>
 
 #include "../../include/moa_attn.h"
 #include "internal.h"
@@ -30,7 +31,28 @@ uint64_t wait_limit_ns() {
 namespace {
 std::mutex g_sm_mu;
 int g_sm_count[64] = {};
+
+struct SmemLimit {
+  const void* func;
+  int dev;
+  int bytes;
+  cudaError_t result;
+};
+std::mutex g_smem_mu;
+std::vector<SmemLimit> g_smem_limits;
 }  // namespace
+
+cudaError_t ensure_smem_limit(const void* func, int bytes) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(g_smem_mu);
+  for (const SmemLimit& s : g_smem_limits)
+    if (s.func == func && s.dev == dev && s.bytes >= bytes) return s.result;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  g_smem_limits.push_back({func, dev, bytes, e});
+  return e;
+}
 
 cudaError_t device_sm_count(int* sms) {
   int dev = -1;

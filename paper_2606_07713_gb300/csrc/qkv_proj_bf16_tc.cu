@@ -19,7 +19,6 @@
 #include <cuda_runtime.h>
 
 #include <cstdio>
-#include <mutex>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -423,15 +422,10 @@ qkv_proj_bf16_mc_kernel(const __grid_constant__ CUtensorMap tmX,
 }  // namespace
 
 int launch_qkv_proj_bf16(const ProjArgs& a, char* msg, size_t msglen) {
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(qkv_proj_bf16_tc_kernel,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(qkv_proj_bf16_mc_kernel,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-  });
+  cudaError_t attr_err =
+      ensure_smem_limit(reinterpret_cast<const void*>(qkv_proj_bf16_tc_kernel), kSmemBytes);
+  if (attr_err == cudaSuccess)
+    attr_err = ensure_smem_limit(reinterpret_cast<const void*>(qkv_proj_bf16_mc_kernel), kSmemBytes);
   if (attr_err != cudaSuccess) {
     snprintf(msg, msglen, "cudaFuncSetAttribute (projection): %s", cudaGetErrorString(attr_err));
     return 5;
