@@ -58,6 +58,7 @@ FP32_SHAPES = [
     (1, 2, 100, 257, 128, 128),
     (1, 1, 1, 1, 4, 4),
     (1, 1, 64, 65, 60, 100),
+    (4, 4, 5, 1000, 32, 96),   # rows of a CTA past N_q; 16 key chunks through the double buffer
 ]
 
 
@@ -102,7 +103,7 @@ def test_bf16_grid_beyond_one_wave(oracle, dk, dv):
 
 def test_fp32_tiled_kernel_on_a_large_grid(oracle):
     """fp32 problems with at least two 32-row CTAs per SM take the tiled kernel (smaller ones take
-    one warp per row); every row checked."""
+    the 8-row small kernel); every row checked."""
     n_sm = torch.cuda.get_device_properties(0).multi_processor_count
     nq = 32 * ((2 * n_sm + 15) // 16)   # 16 heads x nq/32 CTAs >= 2 per SM
     cfg = I.custom_config(2, 8, nq, 300, 64, 64, dtype="fp32", seed=41)
