@@ -113,7 +113,8 @@ def attn_bwd(q, k, v, o, lse, do, scale: float | None = None, workspace=None, st
              fused: bool = False):
     """(dQ, dK, dV) for O = softmax(scale q k^T) v given dO = dL/dO, from the forward's o and lse
     (attn_fwd_lse).  CUDA tensors [B, H, N, d]; lse float32 [B, H, N_q].  fused=True runs
-    moa_attn_bwd_fused (bf16, d_k = d_v = 64; dQ summed with atomics)."""
+    moa_attn_bwd_fused (bf16, d_k = d_v = 64; the key blocks' dQ tiles are added in fp32 by TMA
+    reductions, in a run-dependent order)."""
     import torch
     for t in (q, k, v, o, do, lse):
         if not t.is_cuda or not t.is_contiguous():
