@@ -68,8 +68,11 @@ def test_shift_invariance_through_inputs():
     assert np.max(np.abs(oa - ob)) <= 2e-2 * np.max(np.abs(oa))
 
 
-def test_heads_are_independent_bitwise():
-    x = inputs((2, 3, 300, 400, 128, 128), 9)
+@pytest.mark.parametrize("dk,dv", [(128, 128), (64, 64), (128, 64)])
+def test_heads_are_independent_bitwise(dk, dv):
+    """A (b, h) slice alone gives the bits of the same slice in a batched call (d = 64 runs the
+    one-tile kernel, the others the two-tile kernel)."""
+    x = inputs((2, 3, 300, 400, dk, dv), 9)
     q, k, v = to_device(x)
     o = pkg.attn_fwd(q, k, v)
     for b, h in ((0, 0), (1, 2)):
