@@ -254,9 +254,9 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
  *   workspace_bytes  its size; must be >= moa_attn_splitkv_workspace_bytes(...) with the same
  *                    num_splits (and, for MOA_SPLITS_AUTO, the same current device)
  * MOA_SPLITS_AUTO: the library chooses from the current device's SM count.  When the
- * B*H*ceil(N_q/256) query blocks (one CTA per SM each) leave SMs idle, every block's key axis
- * is split so that the CTAs fill the SMs (at least two key blocks per range), when a model of
- * the split's cost predicts a saving of at least 15 %; with a full wave of blocks or more
+ * B*H*ceil(N_q/256) query blocks (one SM's worth of work each) leave SMs idle, every block's
+ * key axis is split so that the CTAs fill the SMs (at least two key blocks per range), when a
+ * model of the split's cost predicts a saving of at least 15 %; with a full wave of blocks or more
  * nothing is split and the call is moa_attn_fwd (same bits).  moa_attn_split_plan reports
  * the choice.
  * MOA_FP32 has no split form: the call then computes the same result with moa_attn_fwd.
