@@ -63,3 +63,35 @@ def test_oracle_ignores_a_common_score_shift(oracle, shape, seed, shift):
     Qb[:, 0] = np.float32(shift / scale)
     oa, ob = oracle.attn(Qa, K, V, scale), oracle.attn(Qb, K, V, scale)
     assert np.max(np.abs(oa - ob)) <= 1e-12 * (1.0 + np.abs(V).max())
+
+
+@settings(max_examples=15, deadline=None)
+@given(shape=st.tuples(st.integers(1, 3), st.integers(1, 4), st.integers(1, 3), st.integers(1, 3)),
+       seed=st.integers(0, 2**31 - 1), scale=st.floats(-1.5, 1.5, allow_nan=False))
+def test_backward_oracle_matches_decimal_central_differences(oracle, shape, seed, scale):
+    """Every entry of dQ, dK and dV from the backward oracle against a central difference of
+    L = sum(dO * O) in 60-digit decimal arithmetic, on random tiny inputs and scales."""
+    import decimal
+    nq, nk, dk, dv = shape
+    r = np.random.default_rng(seed)
+    f32 = lambda a: np.asarray(a, dtype=np.float32)
+    Q, K = f32(r.normal(size=(nq, dk)) * 1.5), f32(r.normal(size=(nk, dk)))
+    V, G = f32(r.normal(size=(nk, dv))), f32(r.normal(size=(nq, dv)))
+    grads = oracle.attn_bwd(Q, K, V, G, scale)
+    ctx = decimal.Context(prec=60)
+    D = lambda x: decimal.Decimal(float(x))
+    mats = [[[D(x) for x in row] for row in M] for M in (Q, K, V)]
+    g = [[D(x) for x in row] for row in G]
+    sc, h = D(scale), decimal.Decimal("1e-12")
+    for which, grad in enumerate(grads):
+        M = mats[which]
+        for a in range(len(M)):
+            for b in range(len(M[0])):
+                keep = M[a][b]
+                M[a][b] = keep + h
+                lp = oracle_pins._decimal_loss(mats[0], mats[1], mats[2], g, sc, ctx)
+                M[a][b] = keep - h
+                lm = oracle_pins._decimal_loss(mats[0], mats[1], mats[2], g, sc, ctx)
+                M[a][b] = keep
+                fd = float(ctx.divide(ctx.subtract(lp, lm), 2 * h))
+                assert abs(grad[a, b] - fd) <= 1e-12 * max(1.0, abs(fd)), (shape, which, a, b)
