@@ -238,194 +238,11 @@ qkv_proj_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmX,
 }
 
 
-// The same projection with the W tiles shared by the two CTAs of a cluster.  The cluster's CTAs
-// compute two adjacent 128-token blocks of one 256-column block in lockstep (pair item pt ->
-// token blocks 2*(pt / n_ntiles) + rank, column block pt % n_ntiles), so they need the same W
-// tile at every k-step: each CTA loads two of its four 64-column panels and multicasts them to
-// both, halving the L2 traffic for W.  A stage of either CTA is refilled only when both CTAs'
-// tensor cores are done with it: every MMA warp releases a stage to both CTAs' empty barriers
-// (count 2) with a multicast commit.  Clusters are synchronised after the barriers are set up
-// and again before TMEM is freed, once each CTA's tensor core has completed every commit, so
-// that no multicast write or arrival targets a CTA that has left.
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
-qkv_proj_bf16_mc_kernel(const __grid_constant__ CUtensorMap tmX,
-                        const __grid_constant__ CUtensorMap tmW, __nv_bfloat16* __restrict__ Q,
-                        __nv_bfloat16* __restrict__ K, __nv_bfloat16* __restrict__ V, ProjDims p,
-                        int n_pair_items, uint64_t wait_limit_ns) {
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~uintptr_t(1023));
-  const uint32_t sbase = smem_u32(smem);
-  const uint32_t bar0 = smem_u32(smem + kOffBar);
-  auto full_bar = [&](int s) { return bar0 + 8u * s; };
-  auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
-  auto acc_full = [&](int a) { return bar0 + 8u * (2 * kStages + a); };
-  auto acc_empty = [&](int a) { return bar0 + 8u * (2 * kStages + kAccs + a); };
-  const uint32_t drain = bar0 + 8u * (2 * kStages + 2 * kAccs);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc + 4);
-
-  const int warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-  const int rank = int(cluster_ctarank());
-  const int cluster = int(blockIdx.x) >> 1, n_clusters = int(gridDim.x) >> 1;
-  constexpr uint16_t kBoth = 0x3;
-  const WaitCtl wc{abort_flag, wait_limit_ns, 0u, &g_moa_proj_status};
-  auto item_m0 = [&](int pt) { return (2 * (pt / p.n_ntiles) + rank) * kBM; };
-  auto item_c0 = [&](int pt) { return (pt % p.n_ntiles) * kBN; };
-
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), 2);  // both CTAs' tensor cores release every stage
-    }
-    for (int a = 0; a < kAccs; ++a) {
-      mbar_init(acc_full(a), 1);
-      mbar_init(acc_empty(a), kEpiThreads);
-    }
-    mbar_init(drain, 1);
-    *abort_flag = 0;
-    fence_barrier_init();
-  }
-  if (warp == kMmaWarp) {
-    tmem_alloc(smem_u32(tmem_slot), kAccs * kBN);
-    tmem_relinquish();
-  }
-  tc_fence_before_sync();
-  // both CTAs' barriers exist before either multicasts into the other
-  cluster_sync_all();
-  tc_fence_after_sync();
-  const uint32_t tmem = *tmem_slot;
-
-  if (warp == kLoadWarp) {
-    if (lane == 0) {
-      tma_prefetch_desc(&tmX);
-      tma_prefetch_desc(&tmW);
-      int slot = 0;
-      uint32_t phase = 0, issued = 0, issued_phase = 0;
-      bool ok = true;
-      for (int pt = cluster; ok && pt < n_pair_items; pt += n_clusters) {
-        const int m0 = item_m0(pt), c0 = item_c0(pt);
-        for (int kt = 0; kt < p.n_ktiles; ++kt) {
-          if (!wait_bounded(empty_bar(slot), phase ^ 1u, wc)) {
-            ok = false;
-            break;
-          }
-          issued |= 1u << slot;
-          issued_phase = (issued_phase & ~(1u << slot)) | (phase << slot);
-          const uint32_t st = sbase + slot * kStageBytes;
-          // own X tile and both halves of W (this CTA's two panels and the peer's two)
-          mbar_arrive_expect_tx(full_bar(slot), kStageBytes);
-          tma_load_3d(st, &tmX, full_bar(slot), kt * kBK, m0, 0);
-#pragma unroll
-          for (int q = 2 * rank; q < 2 * rank + 2; ++q)
-            tma_load_3d_mc(st + kXBytes + q * kWPanelBytes, &tmW, full_bar(slot), c0 + 64 * q,
-                           kt * kBK, 0, kBoth);
-          if (++slot == kStages) {
-            slot = 0;
-            phase ^= 1u;
-          }
-        }
-      }
-      if (!ok || *abort_flag)
-        for (int sl = 0; sl < kStages; ++sl)
-          if (issued & (1u << sl))
-            wait_quiesce(full_bar(sl), (issued_phase >> sl) & 1u, wait_limit_ns, &g_moa_proj_status);
-    }
-  } else if (warp == kMmaWarp) {
-    if (lane == 0) {
-      constexpr uint32_t kIdesc = make_idesc(kBM, kBN, true);
-      int slot = 0;
-      uint32_t phase = 0;
-      bool ok = true;
-      int it = 0;
-      for (int pt = cluster; ok && pt < n_pair_items; pt += n_clusters, ++it) {
-        const int a = it & 1;
-        const uint32_t tacc = tmem + a * kBN;
-        ok = wait_bounded(acc_empty(a), (uint32_t(it >> 1) & 1u) ^ 1u, wc);
-        if (!ok) break;
-        tc_fence_after_sync();
-        for (int kt = 0; kt < p.n_ktiles; ++kt) {
-          ok = wait_bounded(full_bar(slot), phase, wc);
-          if (!ok) break;
-          tc_fence_after_sync();
-          const uint32_t st = sbase + slot * kStageBytes;
-#pragma unroll
-          for (int kk = 0; kk < kBK / 16; ++kk)
-            mma_f16_ss(tacc, make_sdesc_sw128(st + kk * 32, 16, 1024),
-                       make_sdesc_sw128(st + kXBytes + kk * 2048, kWPanelBytes, 1024), kIdesc,
-                       (kt > 0 || kk > 0) ? 1u : 0u);
-          mma_commit_mc(empty_bar(slot), kBoth);  // this stage is free in both CTAs' view
-          if (++slot == kStages) {
-            slot = 0;
-            phase ^= 1u;
-          }
-        }
-        if (ok) mma_commit(acc_full(a));
-      }
-      mma_commit(drain);  // TMEM quiescent and every earlier commit done, also on the abort path
-    }
-  } else {
-    const int lane_base = (warp & 3) * 32;
-    const int r = lane_base + lane;
-    const int hq = p.H * p.dk;
-    int it = 0;
-    for (int pt = cluster; pt < n_pair_items; pt += n_clusters, ++it) {
-      const int a = it & 1;
-      if (!wait_bounded(acc_full(a), uint32_t(it >> 1) & 1u, wc)) break;
-      tc_fence_after_sync();
-      const int m = item_m0(pt) + r, c0 = item_c0(pt);
-      const bool row_ok = m < p.M;
-      const int b = row_ok ? m / p.N : 0, n = row_ok ? m % p.N : 0;
-#pragma unroll 2
-      for (int c = 0; c < kBN; c += 32) {
-        uint32_t o[32];
-        tmem_ld_32x32b_x32(tmem + (uint32_t(lane_base) << 16) + a * kBN + c, o);
-        tmem_wait_ld();
-        reg_anchor_x32(o);
-        const int col = c0 + c;
-        if (!row_ok || col >= p.ncol) continue;
-        __nv_bfloat16* dst;
-        if (col < hq) {
-          dst = Q + ((size_t(b) * p.H + col / p.dk) * p.N + n) * p.dk + col % p.dk;
-        } else if (col < 2 * hq) {
-          const int cc = col - hq;
-          dst = K + ((size_t(b) * p.H + cc / p.dk) * p.N + n) * p.dk + cc % p.dk;
-        } else {
-          const int cc = col - 2 * hq;
-          dst = V + ((size_t(b) * p.H + cc / p.dv) * p.N + n) * p.dv + cc % p.dv;
-        }
-        uint4 pkt[4];
-        uint32_t* w = reinterpret_cast<uint32_t*>(pkt);
-#pragma unroll
-        for (int i = 0; i < 16; ++i)
-          w[i] = pack_bf16x2(__uint_as_float(o[2 * i]), __uint_as_float(o[2 * i + 1]));
-        uint4* d4 = reinterpret_cast<uint4*>(dst);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) d4[i] = pkt[i];
-      }
-      tc_fence_before_sync();
-      mbar_arrive(acc_empty(a));
-    }
-  }
-
-  if (warp == kMmaWarp) wait_quiesce(drain, 0, wait_limit_ns, &g_moa_proj_status);
-  tc_fence_before_sync();
-  // neither CTA leaves while the other's tensor core or TMA may still reach its shared memory
-  cluster_sync_all();
-  if (warp == kMmaWarp) {
-    tc_fence_after_sync();
-    tmem_dealloc(tmem, kAccs * kBN);
-  }
-}
-
 }  // namespace
 
 int launch_qkv_proj_bf16(const ProjArgs& a, char* msg, size_t msglen) {
   cudaError_t attr_err =
       ensure_smem_limit(reinterpret_cast<const void*>(qkv_proj_bf16_tc_kernel), kSmemBytes);
-  if (attr_err == cudaSuccess)
-    attr_err = ensure_smem_limit(reinterpret_cast<const void*>(qkv_proj_bf16_mc_kernel), kSmemBytes);
   if (attr_err != cudaSuccess) {
     snprintf(msg, msglen, "cudaFuncSetAttribute (projection): %s", cudaGetErrorString(attr_err));
     return 5;
@@ -451,38 +268,6 @@ int launch_qkv_proj_bf16(const ProjArgs& a, char* msg, size_t msglen) {
   // X as [1, M, d] (box 64 x 128 rows); W as [1, d, ncol] (box 64 columns x 64 rows)
   if (!encode_bf16_map_box(&mx, a.X, 1, p.M, a.d, 128, msg, msglen)) return 5;
   if (!encode_bf16_map_box(&mw, a.W, 1, a.d, p.ncol, 64, msg, msglen)) return 5;
-  if (n_mtiles >= 2) {
-    // Clusters of two CTAs sharing the W tiles: as many clusters as can be resident at once.
-    const int64_t n_pair_items = (n_mtiles + 1) / 2 * p.n_ntiles;
-    if (n_pair_items > 0x7fffffffLL) {
-      snprintf(msg, msglen, "projection: too many tiles");
-      return 3;
-    }
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(unsigned(2 * (sm_count / 2)));
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = kSmemBytes;
-    cfg.stream = a.stream;
-    int max_clusters = 0;
-    cudaError_t oe = cudaOccupancyMaxActiveClusters(&max_clusters, qkv_proj_bf16_mc_kernel, &cfg);
-    if (oe != cudaSuccess || max_clusters < 1) {
-      snprintf(msg, msglen, "projection: no resident cluster of two CTAs (%s)",
-               cudaGetErrorString(oe));
-      return 5;
-    }
-    const int64_t clusters = n_pair_items < max_clusters ? n_pair_items : max_clusters;
-    qkv_proj_bf16_mc_kernel<<<dim3(unsigned(2 * clusters)), dim3(kThreads), kSmemBytes,
-                              a.stream>>>(mx, mw, static_cast<__nv_bfloat16*>(a.Q),
-                                          static_cast<__nv_bfloat16*>(a.K),
-                                          static_cast<__nv_bfloat16*>(a.V), p, int(n_pair_items),
-                                          wait_limit_ns());
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) {
-      snprintf(msg, msglen, "projection launch: %s", cudaGetErrorString(e));
-      return 5;
-    }
-    return 0;
-  }
   const int grid = int(n_tiles < sm_count ? n_tiles : sm_count);
   if (n_tiles > 0x7fffffffLL) {
     snprintf(msg, msglen, "projection: too many tiles");
