@@ -1,11 +1,14 @@
 """Benchmark of the DNF attention forward on GB300.
 
-Default workload: bf16 SDPA forward, B=4, H=16, N_q=N_k=2048, d_k=d_v=64, Q/K/V i.i.d.
-N(0,1) from the seeded generator, scale=1/sqrt(d_k), no mask.  One step = one attention
-forward over that batch (the whole hot path: one kernel launch).
+Default workload: the stability stress case, bf16 SDPA forward, B=1, H=16, N_q=N_k=32768,
+d_k=d_v=128, Q/K drawn 8*N(0,1) with 8 planted one-hot rows per head, V ~ N(0,1),
+scale=1/sqrt(d_k), no mask: the largest single-GPU workload, and the paper's long-context length
+(Section 6.2).  One step = one attention forward over that batch (the whole hot path: one kernel
+launch).  `--workload 2` selects the small d=64 case, 3 and 4 the other bf16 shapes, 1 the fp32 one.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference|classical]
                     [--workload ID] [--shape B,H,N_q,N_k,d_k,d_v] [--pass fwd|bwd|qkv]
+                    [--shard bh|replica]
 
 Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s: FLOPs of every step on every
 rank divided by the slowest rank's summed kernel time, measured with CUDA events on the
@@ -19,8 +22,13 @@ elementwise/reduction kernels) -- a measurement of the comparison, not part of t
 `--shape` replaces the workload's sizes (bf16, same generator) for traffic sweeps.  `--pass bwd`
 times moa_attn_bwd (three launches) on the same workload instead of the forward pass, and
 `--pass qkv` the fused projection moa_qkv_proj producing that workload's Q, K, V from an input
-X [B, N, H*d_k].  Multi-GPU (torchrun): every rank runs its own full copy of the workload (the
-(b, h) problems are independent; no collective on the data path), so scaling is weak.
+X [B, N, H*d_k].
+
+Multi-GPU (torchrun), forward pass: by default (`--shard bh`) the workload's B*H independent
+(b, h) slices are partitioned into contiguous ranges, one per rank, and each rank runs the
+forward on its own range only: no collective touches the data (one all_reduce(MAX) of the
+timings), and the total work is fixed, so scaling is strong.  `--shard replica` instead runs the
+whole workload on every rank (weak scaling); the backward and projection passes always do that.
 """
 from __future__ import annotations
 
@@ -43,9 +51,11 @@ import numpy as np  # noqa: E402
 from paper_2606_07713_gb300 import inputs as I  # noqa: E402
 
 METRIC = "attention fwd TFLOP/s and % of GB300 bf16 peak; DRAM bytes vs DNF minimum"
-DEFAULT_WORKLOAD = 2
+DEFAULT_WORKLOAD = 5
 PROFILES = {2: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b4h16n2048d64.txt"),
-            3: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b2h32n8192d128.txt")}
+            3: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b2h32n8192d128.txt"),
+            4: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b8h8nq1024nk4096dk128dv64.txt"),
+            5: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b1h16n32768d128_stress.txt")}
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2606_07713_gb300", "csrc", f)
                   for f in ("attn_fwd_bf16_tc.cu", "ptx.cuh", "tc_common.cuh")]
 FLUSH_BYTES = 256 << 20
@@ -79,38 +89,55 @@ def kernel_source_hash() -> str:
     return h.hexdigest()
 
 
-def profiled_traffic(workload: int) -> tuple[float | None, float | None]:
-    """(DRAM bytes per launch, ncu duration) from the committed ncu summary of this workload,
-    if it was captured from the current kernel source; (None, None) otherwise."""
+def profiled_traffic(workload: int) -> dict | None:
+    """DRAM bytes read and written per launch of the forward kernel, from the committed ncu
+    summary of this workload, if it was captured from the current kernel source; else None."""
     try:
         text = open(PROFILES[workload]).read()
     except (KeyError, OSError):
-        return None, None
+        return None
     m = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", text)
-    b = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
-    if not m or not b or m.group(1) != kernel_source_hash():
-        return None, None
-    return float(b.group(1)), None
+    rd = re.search(r"dram_read_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    wr = re.search(r"dram_write_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    if not m or not rd or not wr or m.group(1) != kernel_source_hash():
+        return None
+    return {"read": float(rd.group(1)), "write": float(wr.group(1))}
+
+
+def traffic_fields(tr: dict | None, dnf: float, o_bytes: float) -> dict:
+    """roofline keys from a profile's DRAM bytes.  `traffic` is ncu's read + write of one launch.
+    A launch can end with part of O still dirty in L2 (written back after the kernel), which
+    would make read + write fall below the DNF minimum; `traffic_vs_dnf` therefore counts the
+    writes as at least |O|: (read + max(write, |O|)) / DNF."""
+    if tr is None:
+        return {"traffic": None, "dram_read": None, "dram_write": None, "traffic_vs_dnf": None}
+    return {"traffic": tr["read"] + tr["write"], "dram_read": tr["read"], "dram_write": tr["write"],
+            "traffic_vs_dnf": round((tr["read"] + max(tr["write"], o_bytes)) / dnf, 4)}
 
 
 class ClockSampler:
-    """nvidia-smi clock/throttle sampling while the timed loop runs."""
+    """nvidia-smi clock/throttle sampling every 20 ms while the timed loops run.  Each sample
+    carries nvidia-smi's own timestamp; mark() records the host-clock windows of the timed loops,
+    and the reported clock statistics use only the samples inside those windows."""
 
-    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,"
+    QUERY = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    PERIOD_MS = 20
+    REASONS = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
 
     def __init__(self, index: int):
         self.index = index
         self.proc = None
         self.lines: list[str] = []
         self.thread = None
+        self.windows: list[tuple[float, float]] = []
 
     def start(self):
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", str(self.PERIOD_MS)],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
@@ -122,9 +149,45 @@ class ClockSampler:
         for line in self.proc.stdout:
             self.lines.append(line.strip())
 
+    def mark(self, t0: float, t1: float) -> None:
+        """A timed window, in time.time() seconds (the host's wall clock)."""
+        self.windows.append((t0, t1))
+
+    @staticmethod
+    def parse(lines, windows, reasons=REASONS) -> dict:
+        """Clock statistics from sample lines (see QUERY) restricted to the windows."""
+        import datetime
+        sm, smax, power, seen, total = [], [], [], set(), 0
+        for ln in lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 10:
+                continue
+            try:
+                t = datetime.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                vals = (float(f[2]), float(f[3]), float(f[4]))
+            except ValueError:
+                continue
+            total += 1
+            if windows and not any(a <= t <= b for a, b in windows):
+                continue
+            sm.append(vals[0])
+            smax.append(vals[1])
+            power.append(vals[2])
+            for n, val in zip(reasons, f[6:10]):
+                if val.lower() == "active":
+                    seen.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "samples": total,
+                    "samples_under_load": 0, "reasons": ["no samples inside the timed loops"]}
+        return {"sm_mhz": float(np.median(sm)), "sm_min_mhz": min(sm), "sm_max_mhz": max(smax),
+                "samples": total, "samples_under_load": len(sm),
+                "period_ms": ClockSampler.PERIOD_MS, "power_w_max": max(power),
+                "reasons": sorted(seen)}
+
     def stop(self) -> dict:
         if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(2 * self.PERIOD_MS / 1000.0)
         self.proc.terminate()
         try:
             self.proc.wait(timeout=5)
@@ -132,25 +195,7 @@ class ClockSampler:
             self.proc.kill()
         if self.thread:
             self.thread.join(timeout=2)
-        sm, smax, reasons, power = [], [], set(), []
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
-            f = [x.strip() for x in ln.split(",")]
-            if len(f) < 9:
-                continue
-            try:
-                sm.append(float(f[1]))
-                smax.append(float(f[2]))
-                power.append(float(f[3]))
-            except ValueError:
-                continue
-            for n, val in zip(names, f[5:9]):
-                if val.lower() == "active":
-                    reasons.add(n)
-        if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
-        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(smax), "samples": len(sm),
-                "power_w_max": max(power) if power else None, "reasons": sorted(reasons)}
+        return self.parse(self.lines, self.windows)
 
 
 def reduce_max_over_ranks(values, device=None):
@@ -168,6 +213,12 @@ def whole_job_tflops(flops_per_step: float, steps: int, world: int, max_ms: floa
     """Weak scaling: every rank runs the full workload, so the job processed world * steps steps
     in the slowest rank's time."""
     return flops_per_step * steps * world / (max_ms * 1e-3) / 1e12
+
+
+def job_tflops(job_flops_per_step: float, steps: int, max_ms: float) -> float:
+    """TFLOP/s of a job whose steps together do job_flops_per_step (over all ranks), timed by
+    the slowest rank."""
+    return job_flops_per_step * steps / (max_ms * 1e-3) / 1e12
 
 
 def to_device_bf16(bits, dev):
@@ -194,6 +245,7 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
     import torch.distributed as dist
 
     import paper_2606_07713_gb300 as pkg
+    from paper_2606_07713_gb300 import shard as SH
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -205,25 +257,43 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
     pkg.lib()
     s = cfg.shape
     x = I.make_inputs(cfg)
+    # This rank's (b, h) slices: a contiguous range of the flattened B*H axis (--shard bh), or
+    # all of them (one GPU, or --shard replica).  A range is one contiguous block of each tensor.
+    bh_total = s.B * s.H
+    sharded = world > 1 and args.shard == "bh"
+    lo, hi = SH.bh_range(bh_total, world, rank) if sharded else (0, bh_total)
+    n_sl = hi - lo
+
+    hb = [SH.block(a, lo, hi) for a in ((x.q_bits, x.k_bits, x.v_bits) if cfg.dtype == "bf16"
+                                         else (x.q, x.k, x.v))]
     if cfg.dtype == "bf16":
-        q, k, v = (to_device_bf16(b, dev) for b in (x.q_bits, x.k_bits, x.v_bits))
-        hq, hk, hv = (torch.from_numpy(np.ascontiguousarray(b).view(np.int16)).view(torch.bfloat16)
-                      .pin_memory() for b in (x.q_bits, x.k_bits, x.v_bits))
+        hq, hk, hv = (torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).pin_memory() for b in hb)
     else:
-        q, k, v = (torch.from_numpy(a).to(dev) for a in (x.q, x.k, x.v))
-        hq, hk, hv = (torch.from_numpy(a).pin_memory() for a in (x.q, x.k, x.v))
-    o = torch.empty((s.B, s.H, s.N_q, s.d_v), dtype=q.dtype, device=dev)
+        hq, hk, hv = (torch.from_numpy(b).pin_memory() for b in hb)
+    q, k, v = (t.to(dev) for t in (hq, hk, hv))
+    o = torch.empty((1, n_sl, s.N_q, s.d_v), dtype=q.dtype, device=dev)
     ho = torch.empty(o.shape, dtype=o.dtype).pin_memory()
     flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
-    flops = pkg.attn_flops(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v)
     code = pkg.MOA_BF16 if cfg.dtype == "bf16" else pkg.MOA_FP32
+    rank_flops = pkg.attn_flops(1, n_sl, s.N_q, s.N_k, s.d_k, s.d_v) if n_sl else 0.0
+    flops = pkg.attn_flops(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v)
+    job_flops = flops if sharded else flops * world
     dnf = pkg.dnf_bytes(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v, code)
+    elt = 2 if cfg.dtype == "bf16" else 4
 
     def barrier():
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize(dev)
+
+    def step(staged: bool):
+        if n_sl == 0:
+            return
+        if staged:
+            pkg.attn_fwd_staged(hq, hk, hv, ho, q, k, v, o, cfg.scale, stream=stream)
+        else:
+            pkg.attn_fwd(q, k, v, cfg.scale, out=o, stream=stream)
 
     # The clock sampler starts first; the warm-up steps then run right before the timed ones,
     # so that the GPU does not idle (and clock down) between them.
@@ -232,20 +302,22 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
     time.sleep(0.3)
     for _ in range(args.warmup):
         flush.zero_()
-        pkg.attn_fwd(q, k, v, cfg.scale, out=o)
+        step(False)
     torch.cuda.synchronize(dev)
     pkg.check(pkg.get_device_status())
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
     barrier()
     t_wall = time.perf_counter()
+    t0 = time.time()
     gpu_head_start(stream)
     for i in range(args.steps):
         flush.zero_()
         ev[i][0].record(stream)
-        pkg.attn_fwd(q, k, v, cfg.scale, out=o, stream=stream)
+        step(False)
         ev[i][1].record(stream)
     barrier()
+    sampler.mark(t0, time.time())
     wall = time.perf_counter() - t_wall
     kern_ms = [a.elapsed_time(b) for a, b in ev]
     total_ms = float(np.sum(kern_ms))
@@ -254,12 +326,14 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
     ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
            for _ in range(args.steps)]
     barrier()
+    t0 = time.time()
     for i in range(args.steps):
         flush.zero_()
         ev2[i][0].record(stream)
-        pkg.attn_fwd_staged(hq, hk, hv, ho, q, k, v, o, cfg.scale, stream=stream)
+        step(True)
         ev2[i][1].record(stream)
     barrier()
+    sampler.mark(t0, time.time())
     clocks = sampler.stop()
     e2e_ms = float(np.sum([a.elapsed_time(b) for a, b in ev2]))
     pkg.check(pkg.get_device_status())
@@ -268,11 +342,16 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
 
     if rank == 0:
         peaks, peak_src = measured_peaks()
-        value = whole_job_tflops(flops, args.steps, world, total_ms)
+        value = job_tflops(job_flops, args.steps, total_ms)
         per_launch_ms = float(np.mean(kern_ms))
-        achieved = flops / (per_launch_ms * 1e-3) / 1e12
+        achieved = rank_flops / (per_launch_ms * 1e-3) / 1e12
         peak = float(peaks["bf16_tflops"]) if cfg.dtype == "bf16" else None
-        traffic, _ = profiled_traffic(cfg.cfg_id)
+        whole_launch = n_sl == bh_total
+        tr = traffic_fields(profiled_traffic(cfg.cfg_id) if whole_launch else None, dnf,
+                            elt * bh_total * s.N_q * s.d_v)
+        in_bytes = elt * bh_total * (s.N_q * s.d_k + s.N_k * s.d_k + s.N_k * s.d_v)
+        out_bytes = elt * bh_total * s.N_q * s.d_v
+        copies = 1 if sharded else world
         line = {
             "metric": METRIC,
             "value": round(value, 2),
@@ -282,11 +361,14 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
             "warmup": args.warmup,
             "ms_per_step": round(total_ms / args.steps, 6),
             "higher_is_better": True,
-            "scaling": "weak",
+            "scaling": "strong" if sharded else "weak",
             "vs_baseline": None,
             "dtype": cfg.dtype,
             "data": "synthetic: seeded splitmix64 + Box-Muller inputs of the workload's shape",
-            "config": workload_desc(cfg),
+            "config": dict(workload_desc(cfg), parallelism=(
+                f"B*H slices partitioned over {world} ranks (contiguous ranges, no data "
+                f"collective)" if sharded else
+                ("one GPU" if world == 1 else f"{world} replicas of the whole workload"))),
             "pct_of_bf16_peak": round(100.0 * achieved / float(peaks["bf16_tflops"]), 2),
             "dnf_bytes": dnf,
             "roofline": {
@@ -296,19 +378,23 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
                 "peak_source": f"{peak_src} bf16_tflops (burst; kernel timed alone)",
                 "unit": "TFLOP/s",
                 "frac": round(achieved / peak, 4) if peak else None,
-                "traffic": traffic,
-                "traffic_vs_dnf": round(traffic / dnf, 4) if traffic else None,
+                **tr,
+                "traffic_source": (os.path.relpath(PROFILES[cfg.cfg_id], ROOT)
+                                   if tr["traffic"] is not None else
+                                   "no ncu summary of this launch from the current kernel source"),
                 "kernel": "attn_fwd_bf16_tc_kernel" if cfg.dtype == "bf16" else "attn_fwd_f32_cc_kernel",
+                "achieved_from": (f"rank 0's launches over {n_sl} of {bh_total} (b, h) slices, "
+                                  "CUDA events on the launching stream"),
             },
             "e2e": {
-                "value": round(whole_job_tflops(flops, args.steps, world, e2e_ms), 2),
+                "value": round(job_tflops(job_flops, args.steps, e2e_ms), 2),
                 "unit": "TFLOP/s",
-                "h2d_bytes_per_step": int(hq.numel() * hq.element_size() + hk.numel() * hk.element_size()
-                                          + hv.numel() * hv.element_size()),
-                "d2h_bytes_per_step": int(ho.numel() * ho.element_size()),
+                "h2d_bytes_per_step": int(in_bytes * copies),
+                "d2h_bytes_per_step": int(out_bytes * copies),
                 "api": "moa_attn_fwd_staged",
             },
-            "gpu_launches": args.steps,
+            # one kernel per step on every rank that owns at least one slice
+            "gpu_launches": args.steps * (min(world, bh_total) if sharded else world),
             "clocks": clocks,
             "wall_s_timed_loop": round(wall, 4),
         }
@@ -417,6 +503,7 @@ def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
     barrier()
+    t0 = time.time()
     gpu_head_start(stream)
     for i in range(args.steps):
         flush.zero_()
@@ -424,6 +511,7 @@ def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
         pkg.attn_bwd(q, k, v, o, lse, do, cfg.scale, workspace=ws, stream=stream, fused=fused)
         ev[i][1].record(stream)
     barrier()
+    sampler.mark(t0, time.time())
     kern_ms = [a.elapsed_time(b) for a, b in ev]
     total_ms = float(np.sum(kern_ms))
     # end to end: the forward's outputs and dO from pinned host memory, gradients back
@@ -432,6 +520,7 @@ def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
     ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
            for _ in range(args.steps)]
     barrier()
+    t0 = time.time()
     for i in range(args.steps):
         flush.zero_()
         ev2[i][0].record(stream)
@@ -443,6 +532,7 @@ def run_ours_bwd(args, cfg: I.AttnConfig) -> None:
             h_.copy_(d_, non_blocking=True)
         ev2[i][1].record(stream)
     barrier()
+    sampler.mark(t0, time.time())
     clocks = sampler.stop()
     e2e_ms = float(np.sum([a.elapsed_time(b) for a, b in ev2]))
     pkg.check(pkg.get_device_status())
@@ -551,6 +641,7 @@ def run_ours_qkv(args, cfg: I.AttnConfig) -> None:
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
     barrier()
+    t0 = time.time()
     gpu_head_start(stream)
     for i in range(args.steps):
         flush.zero_()
@@ -558,11 +649,13 @@ def run_ours_qkv(args, cfg: I.AttnConfig) -> None:
         pkg.qkv_proj(x, w, s.H, s.d_k, s.d_v, out=(q, k, v), stream=stream)
         ev[i][1].record(stream)
     barrier()
+    sampler.mark(t0, time.time())
     kern_ms = [a.elapsed_time(b) for a, b in ev]
     total_ms = float(np.sum(kern_ms))
     ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
            for _ in range(args.steps)]
     barrier()
+    t0 = time.time()
     for i in range(args.steps):
         flush.zero_()
         ev2[i][0].record(stream)
@@ -573,6 +666,7 @@ def run_ours_qkv(args, cfg: I.AttnConfig) -> None:
             h_.copy_(d_, non_blocking=True)
         ev2[i][1].record(stream)
     barrier()
+    sampler.mark(t0, time.time())
     clocks = sampler.stop()
     e2e_ms = float(np.sum([a.elapsed_time(b) for a, b in ev2]))
     pkg.check(pkg.get_device_status())
@@ -793,15 +887,19 @@ def run_reference(args, cfg: I.AttnConfig) -> None:
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference", "classical"], default="ours")
     ap.add_argument("--workload", type=int, default=DEFAULT_WORKLOAD, choices=sorted(I.CONFIGS))
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle time for the cpu_baseline sample")
     ap.add_argument("--bwd-path", choices=["auto", "fused", "split"], default="auto",
-                    help="backward kernels: fused (one tile kernel, d_k = d_v = 64), split (dK/dV "
-                         "and dQ kernels), auto (fused where it applies)")
+                    help="backward kernels: fused (one tile kernel, d_k = d_v = 64; its dQ is not "
+                         "bitwise reproducible), split (dK/dV and dQ kernels; bitwise "
+                         "reproducible), auto (fused where it applies)")
+    ap.add_argument("--shard", choices=["bh", "replica"], default="bh",
+                    help="forward pass on N > 1 GPUs: bh partitions the B*H slices over the ranks "
+                         "(strong scaling), replica runs the whole workload on every rank (weak)")
     ap.add_argument("--pass", dest="which", choices=["fwd", "bwd", "qkv"], default="fwd",
                     help="time the forward (default), the backward pass or the QKV projection")
     ap.add_argument("--shape", default=None,

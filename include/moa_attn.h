@@ -165,8 +165,9 @@ size_t moa_attn_bwd_workspace_bytes(int64_t B, int64_t H, int64_t N_q, int64_t N
  * dtype MOA_BF16 and d_k = d_v = 64 only, and a workspace of at least
  * moa_attn_bwd_fused_workspace_bytes(...) bytes.
  * Reproducibility: dK and dV are bitwise reproducible; the order of the fp32 additions into dQ
- * varies between runs, so dQ may differ in its last bits from run to run (moa_attn_bwd's dQ
- * does not).
+ * varies between runs, so dQ may differ in its last bits from run to run.  Callers that need
+ * bit-identical gradients from identical inputs call moa_attn_bwd, whose three gradients are
+ * all bitwise reproducible.
  * Errors: those of moa_attn_bwd; MOA_ERR_UNSUPPORTED_DTYPE for fp32, MOA_ERR_UNSUPPORTED_SHAPE
  * for other head dimensions.
  * Behaviour: asynchronous; three kernel launches on `stream` (per-row D and LSE with the

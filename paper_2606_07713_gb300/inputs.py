@@ -19,6 +19,13 @@ Generator (all in float64, vectorised with numpy):
 
 Streams: Q = 0, K = 1, V = 2, planted rows = 3.
 
+Planted rows (the stability workload): per head, distinct query rows i_r and distinct keys k_r
+are drawn from stream 3, and Q[i_r] is set to the stored K[k_r].  A drawn key is kept only if,
+in float64 on the stored values, the row's score for k_r beats every other key's score by more
+than PLANT_MARGIN (scores are scale * <q, k>); otherwise the next key is drawn from the same
+stream.  This inner product is the input recipe's acceptance test, not an attention step: both
+the oracle and the kernels receive the finished arrays.
+
 The five workload shapes follow the paper's problem statement (Section 4.1,
 Eq. attention, with the batched/multi-head layout of the Remark in Section 4.2):
 Q [B,H,N_q,d_k], K [B,H,N_k,d_k], V [B,H,N_k,d_v], contiguous row-major.
@@ -39,6 +46,9 @@ _M2 = np.uint64(0x94D049BB133111EB)
 _CHUNK = 1 << 20
 
 STREAM_Q, STREAM_K, STREAM_V, STREAM_PLANT, STREAM_DO = 0, 1, 2, 3, 4
+
+PLANT_MARGIN = 30.0     # a planted key's score must beat the row's next best by more than this
+PLANT_MAX_DRAWS = 64    # key candidates drawn per planted row before the recipe gives up
 
 
 def _mix64(z: np.ndarray) -> np.ndarray:
@@ -199,6 +209,7 @@ class AttnInputs:
     k_bits: Optional[np.ndarray] = None
     v_bits: Optional[np.ndarray] = None
     plants: tuple = ()
+    plant_redraws: int = 0     # key candidates rejected by the margin rule
 
     @property
     def shape(self) -> AttnShape:
@@ -228,6 +239,35 @@ def _distinct_indices(seed: int, stream: int, start: int, n: int, limit: int):
         if c not in chosen:
             chosen.append(c)
     return chosen, pos
+
+
+def _plant_keys(seed: int, start: int, k_head: np.ndarray, n: int, scale: float):
+    """n distinct keys of one head for planted rows, drawn in order from the plant stream.  A
+    candidate c is accepted when scale * <K[c], K[c]> exceeds scale * <K[c], K[j]> for every other
+    key j by more than PLANT_MARGIN (float64 on the stored values); duplicates and candidates
+    short of the margin are skipped.  Returns (keys, next stream position, rejected count)."""
+    n_k = k_head.shape[0]
+    kh = np.asarray(k_head, dtype=np.float64)
+    chosen: list[int] = []
+    pos, rejected = start, 0
+    for _ in range(n):
+        for _attempt in range(PLANT_MAX_DRAWS):
+            u = uniform01(seed, STREAM_PLANT, pos, 1)[0]
+            pos += 1
+            c = min(int(u * n_k), n_k - 1)
+            if c in chosen:
+                continue
+            sc = scale * (kh @ kh[c])
+            own = sc[c]
+            sc[c] = -np.inf
+            if n_k == 1 or own - np.max(sc) > PLANT_MARGIN:
+                chosen.append(c)
+                break
+            rejected += 1
+        else:
+            raise ValueError(f"no key with a score margin above {PLANT_MARGIN} in "
+                             f"{PLANT_MAX_DRAWS} draws: this head cannot host a planted row")
+    return chosen, pos, rejected
 
 
 def make_inputs(cfg: AttnConfig | int) -> AttnInputs:
@@ -261,6 +301,7 @@ def make_inputs(cfg: AttnConfig | int) -> AttnInputs:
         kb = kb.reshape(k.shape)
         vb = vb.reshape(v.shape)
     plants = []
+    redraws = 0
     if cfg.plants_per_head:
         if s.N_q < cfg.plants_per_head or s.N_k < cfg.plants_per_head:
             raise ValueError("plants need N_q, N_k >= plants_per_head")
@@ -268,13 +309,14 @@ def make_inputs(cfg: AttnConfig | int) -> AttnInputs:
         for b in range(s.B):
             for h in range(s.H):
                 rows, pos = _distinct_indices(seed, STREAM_PLANT, pos, cfg.plants_per_head, s.N_q)
-                keys, pos = _distinct_indices(seed, STREAM_PLANT, pos, cfg.plants_per_head, s.N_k)
+                keys, pos, rej = _plant_keys(seed, pos, k[b, h], len(rows), cfg.scale)
+                redraws += rej
                 for i, kk in zip(rows, keys):
                     q[b, h, i, :] = k[b, h, kk, :]
                     if qb is not None:
                         qb[b, h, i, :] = kb[b, h, kk, :]
                     plants.append((b, h, i, kk))
-    return AttnInputs(cfg, q, k, v, qb, kb, vb, tuple(plants))
+    return AttnInputs(cfg, q, k, v, qb, kb, vb, tuple(plants), redraws)
 
 
 def make_grad_output(cfg: AttnConfig | int, sigma: float = 1.0):

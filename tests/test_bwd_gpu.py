@@ -173,3 +173,22 @@ def test_bwd_d128_workload_sampled_head(oracle):
                           g[b:b + 1, h:h + 1], x.scale)
     got = tuple(t[b:b + 1, h:h + 1] for t in (dq, dk, dv))
     check_grads(got, ref, f"workload 3 slice ({b},{h})")
+
+
+@pytest.mark.parametrize("dtype,dk,dv", [("bf16", 64, 64), ("bf16", 128, 128), ("bf16", 128, 64),
+                                         ("fp32", 64, 64)])
+def test_three_kernel_backward_bitwise_reproducible(dtype, dk, dv):
+    """moa_attn_bwd adds every gradient in a fixed order, so two calls on the same inputs give
+    the same bits (the reproducible choice; moa_attn_bwd_fused's dQ is not)."""
+    cfg = I.custom_config(2, 4, 700, 900, dk, dv, dtype=dtype, seed=dk + dv)
+    x = I.make_inputs(cfg)
+    g, gb = I.make_grad_output(cfg)
+    q, k, v = to_device(x)
+    do = bf16_dev(gb) if dtype == "bf16" else torch.from_numpy(np.ascontiguousarray(g)).to("cuda:0")
+    o, lse = pkg.attn_fwd_lse(q, k, v, x.scale)
+    a = pkg.attn_bwd(q, k, v, o, lse, do, x.scale)
+    b = pkg.attn_bwd(q, k, v, o, lse, do, x.scale)
+    torch.cuda.synchronize()
+    pkg.check(pkg.get_device_status())
+    for name, ta, tb in zip(("dQ", "dK", "dV"), a, b):
+        assert torch.equal(ta, tb), name

@@ -66,3 +66,47 @@ def test_five_workloads_declared():
     s = I.CONFIGS[4].shape
     assert (s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v) == (8, 8, 1024, 4096, 128, 64)
     assert I.CONFIGS[1].dtype == "fp32" and I.CONFIGS[5].plants_per_head == 8
+
+
+def _margins(oracle, x):
+    """Score margin of every planted row over its next-best key, from the oracle's scores."""
+    out = []
+    for (b, h, i, kk) in x.plants:
+        sc = oracle.scores(x.q[b, h, i:i + 1], x.k[b, h], x.scale)[0]
+        own = sc[kk]
+        sc[kk] = -np.inf
+        out.append(own - np.max(sc))
+    return np.array(out)
+
+
+def test_plant_keys_redrawn_until_margin(oracle):
+    # Q, K ~ 2.5 N(0,1), d = 64, 1024 keys: a planted score is about 50 +- 9 and the next best
+    # about 20, so roughly half of the first candidates fall short of the margin and are redrawn.
+    cfg = I.custom_config(1, 3, 64, 1024, 64, 64, dtype="bf16", seed=9, q_sigma=2.5, k_sigma=2.5,
+                          plants_per_head=4)
+    x = I.make_inputs(cfg)
+    assert x.plant_redraws > 0
+    assert np.all(_margins(oracle, x) > I.PLANT_MARGIN)
+    for h in range(3):
+        keys = [kk for (_, hh, _, kk) in x.plants if hh == h]
+        rows = [i for (_, hh, i, _) in x.plants if hh == h]
+        assert len(set(keys)) == 4 and len(set(rows)) == 4
+    # the redraws come from the seeded stream, so the plants are reproducible
+    y = I.make_inputs(I.custom_config(1, 3, 64, 1024, 64, 64, dtype="bf16", seed=9,
+                                      q_sigma=2.5, k_sigma=2.5, plants_per_head=4))
+    assert y.plants == x.plants
+
+
+def test_plant_margin_holds_for_stress_shape(oracle):
+    # the stability workload's distributions (sigma 8, d = 128) at a smaller key count
+    cfg = I.custom_config(1, 2, 256, 4096, 128, 128, dtype="bf16", seed=5, q_sigma=8.0,
+                          k_sigma=8.0, plants_per_head=8)
+    x = I.make_inputs(cfg)
+    assert len(x.plants) == 16 and np.all(_margins(oracle, x) > I.PLANT_MARGIN)
+
+
+def test_plant_without_any_margin_is_refused():
+    # d = 8, unit scale: a planted score is about 2.8, far below the margin for every key
+    cfg = I.custom_config(1, 1, 16, 64, 8, 8, dtype="fp32", seed=3, plants_per_head=1)
+    with pytest.raises(ValueError, match="margin"):
+        I.make_inputs(cfg)

@@ -81,6 +81,27 @@ def test_heads_are_independent_bitwise(dk, dv):
         assert torch.equal(one[0, 0], o[b, h])
 
 
+@pytest.mark.parametrize("dk,dv,dtype", [(128, 128, "bf16"), (64, 64, "bf16"), (128, 64, "bf16"),
+                                         (64, 64, "fp32")])
+@pytest.mark.parametrize("world", [2, 3, 5])
+def test_bh_ranges_reassemble_the_whole_call_bitwise(dk, dv, dtype, world):
+    """The multi-GPU partition on one GPU: each rank's call runs on its contiguous block of
+    (b, h) slices through pointer offsets into the same tensors (shard.block_view), writing its
+    block of O in place; together the calls give the whole call's bits.  B*H = 14 is not a
+    multiple of any of the rank counts."""
+    from paper_2606_07713_gb300 import shard as SH
+    x = inputs((2, 7, 300, 400, dk, dv), 19 + dk, dtype)
+    q, k, v = to_device(x)
+    whole = pkg.attn_fwd(q, k, v)
+    parts = torch.full_like(whole, float("nan"))
+    for lo, hi in SH.bh_ranges(14, world):
+        pkg.attn_fwd(SH.block_view(q, lo, hi), SH.block_view(k, lo, hi), SH.block_view(v, lo, hi),
+                     out=SH.block_view(parts, lo, hi))
+    torch.cuda.synchronize()
+    pkg.check(pkg.get_device_status())
+    assert torch.equal(parts, whole)
+
+
 @pytest.mark.parametrize("dtype", ["bf16", "fp32"])
 def test_run_to_run_bitwise_deterministic(dtype):
     x = inputs((2, 4, 1000, 1500, 64, 64), 10, dtype)

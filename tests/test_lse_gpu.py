@@ -8,7 +8,7 @@ exp2/log2 (bf16 path: MUFU, about 2^-22) and of the final multiply by ln 2.
 import numpy as np
 import pytest
 
-from gpu_helpers import assert_close, to_device
+from gpu_helpers import assert_close, lse_bound, to_device
 
 pytestmark = pytest.mark.gpu
 
@@ -23,15 +23,6 @@ def _need_gpu():
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     pkg.lib()
-
-
-def lse_bound(x, lse_ref, scale=None):
-    scale = x.scale if scale is None else scale
-    q = np.abs(x.q.astype(np.float64))
-    k = np.abs(x.k.astype(np.float64))
-    dk = x.q.shape[-1]
-    score_err = dk * 2.0 ** -24 * abs(scale) * np.max(q @ np.swapaxes(k, -1, -2), axis=-1)
-    return 4.0 * score_err + 4e-6 * (1.0 + np.abs(lse_ref))
 
 
 def run_lse(x, scale=None):

@@ -56,9 +56,51 @@ def test_noalloc_matches_workspace_entry_point_on_consecutive_calls():
                                                    _lib.MOA_BF16, splits, stream)
             assert rc == _lib.MOA_OK, _lib.moa_last_error()
             torch.cuda.synchronize()
+            # the same split and merge kernels on the same plan: the same bits, so a partial left
+            # in the scratch by the previous call cannot hide inside a tolerance
+            assert torch.equal(o, o_ref), (shape, call)
             got = o.float().cpu().numpy()
             want = o_ref.float().cpu().numpy()
             assert np.all(np.isfinite(got)), (shape, call)
             err = float(np.max(np.abs(got - want)) / np.max(np.abs(want)))
             assert err <= BF16_TOL, (shape, call, err)
+    assert _lib.moa_get_device_status(stream) == _lib.MOA_OK
+
+
+@pytest.mark.gpu
+def test_noalloc_automatic_split_too_large_for_the_scratch_runs_unsplit():
+    """With MOA_SPLITS_AUTO the library's own choice never fails for want of scratch: when the
+    automatic plan's partials would not fit the static array, the call runs unsplit and gives
+    moa_attn_fwd's bits."""
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from gpu_helpers import to_device
+    _lib.lib()
+    stream = torch.cuda.current_stream().cuda_stream
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    # 64 heads x one 256-row query block = 64 blocks < the SM count: the automatic plan splits
+    # every block's 16 key blocks in two, whose partials (2 x 16384 rows x 520 bytes, 17.0 MB)
+    # exceed the 16 MiB array.
+    shape = (1, 64, 256, 2048, 128, 128)
+    B, H, Nq, Nk, dk, dv = shape
+    rc, n_splits, _, _ = _lib.moa_attn_split_plan(B, H, Nq, Nk, _lib.MOA_SPLITS_AUTO, sms)
+    assert rc == _lib.MOA_OK and n_splits > 1
+    need = n_splits * B * H * Nq * (4 * dv + 8)
+    assert need > _lib.MOA_NOALLOC_SCRATCH_BYTES
+    x = I.make_inputs(I.custom_config(*shape, dtype="bf16", seed=23))
+    q, k, v = to_device(x)
+    scale = ctypes.c_float(x.scale).value
+    o_ref = torch.empty((B, H, Nq, dv), dtype=torch.bfloat16, device=q.device)
+    rc = _lib.moa_attn_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), o_ref.data_ptr(), B, H, Nq,
+                           Nk, dk, dv, scale, _lib.MOA_BF16, stream)
+    assert rc == _lib.MOA_OK, _lib.moa_last_error()
+    for call in range(2):
+        o = torch.full_like(o_ref, float("nan"))
+        rc = _lib.moa_attn_fwd_splitkv_noalloc(q.data_ptr(), k.data_ptr(), v.data_ptr(),
+                                               o.data_ptr(), B, H, Nq, Nk, dk, dv, scale,
+                                               _lib.MOA_BF16, _lib.MOA_SPLITS_AUTO, stream)
+        assert rc == _lib.MOA_OK, _lib.moa_last_error()
+        torch.cuda.synchronize()
+        assert torch.equal(o, o_ref), call
     assert _lib.moa_get_device_status(stream) == _lib.MOA_OK
