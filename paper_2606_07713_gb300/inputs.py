@@ -19,11 +19,11 @@ Generator (all in float64, vectorised with numpy):
 
 Streams: Q = 0, K = 1, V = 2, planted rows = 3.
 
-Planted rows (the stability workload): per head, distinct query rows i_r and distinct keys k_r
-are drawn from stream 3, and Q[i_r] is set to the stored K[k_r].  A drawn key is kept only if,
-in float64 on the stored values, the row's score for k_r beats every other key's score by more
-than PLANT_MARGIN (scores are scale * <q, k>); otherwise the next key is drawn from the same
-stream.  This inner product is the input recipe's acceptance test, not an attention step: both
+Planted rows: per head, distinct query rows i_r and distinct keys k_r are drawn from stream 3,
+and Q[i_r] is set to the stored K[k_r].  With a plant margin (the stability workload uses
+PLANT_MARGIN), a drawn key is kept only if, in float64 on the stored values, the row's score for
+k_r beats every other key's score by more than the margin (scores are scale * <q, k>);
+otherwise the next key is drawn from the same stream.  This inner product is the input recipe's acceptance test, not an attention step: both
 the oracle and the kernels receive the finished arrays.
 
 The five workload shapes follow the paper's problem statement (Section 4.1,
@@ -168,7 +168,9 @@ class AttnConfig:
     q_sigma: float = 1.0       # Q ~ q_sigma * N(0,1)
     k_sigma: float = 1.0       # K ~ k_sigma * N(0,1)
     v_dist: str = "normal"     # "normal" -> N(0,1); "uniform" -> U[-1,1]
-    plants_per_head: int = 0   # rows i with Q[i] := K[k*] (one dominant key)
+    plants_per_head: int = 0   # rows i with Q[i] := K[k*]
+    # planted key must beat the row's next best score by more than this (None: any key)
+    plant_margin: Optional[float] = None
     seed: Optional[int] = None
 
     @property
@@ -189,7 +191,7 @@ CONFIGS = {
                   "bf16", v_dist="uniform"),
     5: AttnConfig(5, "bf16 B1 H16 N32768 d128 stress (QK sigma 8, planted rows)",
                   AttnShape(1, 16, 32768, 32768, 128, 128), "bf16",
-                  q_sigma=8.0, k_sigma=8.0, plants_per_head=8),
+                  q_sigma=8.0, k_sigma=8.0, plants_per_head=8, plant_margin=PLANT_MARGIN),
 }
 
 
@@ -241,13 +243,15 @@ def _distinct_indices(seed: int, stream: int, start: int, n: int, limit: int):
     return chosen, pos
 
 
-def _plant_keys(seed: int, start: int, k_head: np.ndarray, n: int, scale: float):
-    """n distinct keys of one head for planted rows, drawn in order from the plant stream.  A
-    candidate c is accepted when scale * <K[c], K[c]> exceeds scale * <K[c], K[j]> for every other
-    key j by more than PLANT_MARGIN (float64 on the stored values); duplicates and candidates
-    short of the margin are skipped.  Returns (keys, next stream position, rejected count)."""
+def _plant_keys(seed: int, start: int, k_head: np.ndarray, n: int, scale: float,
+                margin: Optional[float]):
+    """n distinct keys of one head for planted rows, drawn in order from the plant stream.  With a
+    margin, a candidate c is accepted only when scale * <K[c], K[c]> exceeds scale * <K[c], K[j]>
+    for every other key j by more than `margin` (float64 on the stored values); duplicates and
+    candidates short of the margin are skipped.  Returns (keys, next stream position, rejected
+    count)."""
     n_k = k_head.shape[0]
-    kh = np.asarray(k_head, dtype=np.float64)
+    kh = np.asarray(k_head, dtype=np.float64) if margin is not None else None
     chosen: list[int] = []
     pos, rejected = start, 0
     for _ in range(n):
@@ -257,15 +261,18 @@ def _plant_keys(seed: int, start: int, k_head: np.ndarray, n: int, scale: float)
             c = min(int(u * n_k), n_k - 1)
             if c in chosen:
                 continue
+            if margin is None:
+                chosen.append(c)
+                break
             sc = scale * (kh @ kh[c])
             own = sc[c]
             sc[c] = -np.inf
-            if n_k == 1 or own - np.max(sc) > PLANT_MARGIN:
+            if n_k == 1 or own - np.max(sc) > margin:
                 chosen.append(c)
                 break
             rejected += 1
         else:
-            raise ValueError(f"no key with a score margin above {PLANT_MARGIN} in "
+            raise ValueError(f"no key with a score margin above {margin} in "
                              f"{PLANT_MAX_DRAWS} draws: this head cannot host a planted row")
     return chosen, pos, rejected
 
@@ -309,7 +316,8 @@ def make_inputs(cfg: AttnConfig | int) -> AttnInputs:
         for b in range(s.B):
             for h in range(s.H):
                 rows, pos = _distinct_indices(seed, STREAM_PLANT, pos, cfg.plants_per_head, s.N_q)
-                keys, pos, rej = _plant_keys(seed, pos, k[b, h], len(rows), cfg.scale)
+                keys, pos, rej = _plant_keys(seed, pos, k[b, h], len(rows), cfg.scale,
+                                             cfg.plant_margin)
                 redraws += rej
                 for i, kk in zip(rows, keys):
                     q[b, h, i, :] = k[b, h, kk, :]
@@ -334,9 +342,10 @@ def make_grad_output(cfg: AttnConfig | int, sigma: float = 1.0):
 
 
 def custom_config(B, H, N_q, N_k, d_k, d_v, dtype="bf16", seed=1234, q_sigma=1.0,
-                  k_sigma=1.0, v_dist="normal", plants_per_head=0) -> AttnConfig:
+                  k_sigma=1.0, v_dist="normal", plants_per_head=0,
+                  plant_margin=None) -> AttnConfig:
     """A workload of any shape with the same generator (used by tests)."""
     return AttnConfig(0, f"custom {dtype} B{B} H{H} Nq{N_q} Nk{N_k} dk{d_k} dv{d_v}",
                       AttnShape(B, H, N_q, N_k, d_k, d_v), dtype, q_sigma=q_sigma,
                       k_sigma=k_sigma, v_dist=v_dist, plants_per_head=plants_per_head,
-                      seed=seed)
+                      plant_margin=plant_margin, seed=seed)

@@ -61,6 +61,11 @@ def test_plants_copy_key_rows():
     assert len(rows) == 12
 
 
+def test_stress_workload_declares_the_margin():
+    assert I.CONFIGS[5].plant_margin == I.PLANT_MARGIN == 30.0
+    assert all(I.CONFIGS[c].plant_margin is None for c in (1, 2, 3, 4))
+
+
 def test_five_workloads_declared():
     assert sorted(I.CONFIGS) == [1, 2, 3, 4, 5]
     s = I.CONFIGS[4].shape
@@ -83,7 +88,7 @@ def test_plant_keys_redrawn_until_margin(oracle):
     # Q, K ~ 2.5 N(0,1), d = 64, 1024 keys: a planted score is about 50 +- 9 and the next best
     # about 20, so roughly half of the first candidates fall short of the margin and are redrawn.
     cfg = I.custom_config(1, 3, 64, 1024, 64, 64, dtype="bf16", seed=9, q_sigma=2.5, k_sigma=2.5,
-                          plants_per_head=4)
+                          plants_per_head=4, plant_margin=I.PLANT_MARGIN)
     x = I.make_inputs(cfg)
     assert x.plant_redraws > 0
     assert np.all(_margins(oracle, x) > I.PLANT_MARGIN)
@@ -92,21 +97,25 @@ def test_plant_keys_redrawn_until_margin(oracle):
         rows = [i for (_, hh, i, _) in x.plants if hh == h]
         assert len(set(keys)) == 4 and len(set(rows)) == 4
     # the redraws come from the seeded stream, so the plants are reproducible
-    y = I.make_inputs(I.custom_config(1, 3, 64, 1024, 64, 64, dtype="bf16", seed=9,
-                                      q_sigma=2.5, k_sigma=2.5, plants_per_head=4))
+    y = I.make_inputs(cfg)
     assert y.plants == x.plants
+    # without a margin the first distinct candidates are kept, some of them short of it
+    z = I.make_inputs(I.custom_config(1, 3, 64, 1024, 64, 64, dtype="bf16", seed=9, q_sigma=2.5,
+                                      k_sigma=2.5, plants_per_head=4))
+    assert z.plant_redraws == 0 and np.min(_margins(oracle, z)) < I.PLANT_MARGIN
 
 
 def test_plant_margin_holds_for_stress_shape(oracle):
     # the stability workload's distributions (sigma 8, d = 128) at a smaller key count
     cfg = I.custom_config(1, 2, 256, 4096, 128, 128, dtype="bf16", seed=5, q_sigma=8.0,
-                          k_sigma=8.0, plants_per_head=8)
+                          k_sigma=8.0, plants_per_head=8, plant_margin=I.PLANT_MARGIN)
     x = I.make_inputs(cfg)
     assert len(x.plants) == 16 and np.all(_margins(oracle, x) > I.PLANT_MARGIN)
 
 
 def test_plant_without_any_margin_is_refused():
     # d = 8, unit scale: a planted score is about 2.8, far below the margin for every key
-    cfg = I.custom_config(1, 1, 16, 64, 8, 8, dtype="fp32", seed=3, plants_per_head=1)
+    cfg = I.custom_config(1, 1, 16, 64, 8, 8, dtype="fp32", seed=3, plants_per_head=1,
+                          plant_margin=I.PLANT_MARGIN)
     with pytest.raises(ValueError, match="margin"):
         I.make_inputs(cfg)
