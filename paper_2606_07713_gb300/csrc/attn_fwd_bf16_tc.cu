@@ -14,30 +14,29 @@
 //     exceeds m by more than kRescaleLog2 (in log2 units), m is raised and O and l are
 //     rescaled by exp2(m_old - m_new); otherwise the stale m is kept.  Both are exact: O and l
 //     always share the same reference maximum, and exponentials stay <= 2^kRescaleLog2.
-//   * The unnormalised probabilities P are rounded to bf16 and written back into the TMEM
-//     columns of S, from where the second tensor-core product O += P V (Eq. output_dnf) reads
-//     them directly.  V is the "MN-major" B operand, again as stored.
+//   * The unnormalised probabilities P are rounded to bf16 and stored where the second
+//     tensor-core product O += P V (Eq. output_dnf) reads them: TMEM columns of their own
+//     (d_v = 64) or a 32 KB shared-memory tile per Q tile (d_v = 128, where S and O fill the
+//     TMEM).  V is the "MN-major" B operand, again as stored.
 //   * Step IV (division, Section 4.5) is applied once per row in the epilogue: O / l.
 //
-// CTA organisation, two-tile kernel (one CTA per SM: 512 TMEM columns, up to ~192 KB shared
+// CTA organisation, two-tile kernel (one CTA per SM: 512 TMEM columns, up to ~225 KB shared
 // memory):
 //   work item = (b*H + h, block of 256 query rows) = two 128-row Q tiles;
 //   warps 0-3: softmax + epilogue of Q tile 0; warps 4-7: same for Q tile 1
 //              (thread t of such a warpgroup owns query row t of its tile);
-//   warp 8:    TMEM allocation; issues tcgen05.mma (both tiles, or tile 0 only, see below);
+//   warp 8:    TMEM allocation; issues the tcgen05.mma products of Q tile 0;
 //   warp 9:    the single thread that issues all TMA loads;
-//   warp 10:   issues tcgen05.mma for tile 1 when P has TMEM columns of its own.
+//   warp 10:   issues the tcgen05.mma products of Q tile 1.
 // One-tile kernel (d_k = d_v = 64 without a split key axis; two CTAs per SM, 256 TMEM columns
 // and ~98 KB of shared memory each): work item = (b*H + h, block of 128 query rows); warps 0-3
 // softmax + epilogue, warp 4 TMEM allocation and tcgen05.mma, warp 5 TMA loads.
-// K and V tiles of 128 keys stream through an NS-stage shared-memory ring.  Two schedules:
-//   d_v = 128 (TMEM: S0 S1 O0 O1): P_j is written over S_j's columns, so per key tile n >= 1
-//     the single issuing thread runs O_j += P_j(n-1) V(n-1) and then S_j = Q_j K(n)^T, tile 0
-//     then tile 1; ring order K0 V0 K1 V1 ...
-//   d_v = 64 (TMEM: S0 S1 P0 P1 O0 O1, one tile: S0 P0 O0): P_j has columns of its own.  As soon as the softmax has
-//     read S_j(n) into registers, tile j's issuing thread computes S_j(n+1), and it runs
-//     O_j += P_j(n) V(n) once P_j(n) is written, so the softmax never waits for the product
-//     with V; ring order K0 K1 V0 K2 V1 ...
+// K and V tiles of 128 keys stream through an NS-stage shared-memory ring.  One schedule: P_j
+// has a buffer of its own (TMEM S0 S1 P0 P1 O0 O1 at d_v = 64, one tile: S0 P0 O0; TMEM
+// S0 S1 O0 O1 plus P0 P1 in shared memory at d_v = 128).  As soon as the softmax has read
+// S_j(n) into registers, tile j's issuing thread computes S_j(n+1), and it runs
+// O_j += P_j(n) V(n) once P_j(n) is written, so the softmax never waits for the product with
+// V; ring order K0 K1 V0 K2 V1 ...
 // TMEM lane = row of the Q tile.
 
 // Every mbarrier wait is bounded (globaltimer); on expiry the kernel records
@@ -95,18 +94,23 @@ struct Cfg {
   static constexpr int kKTileBytes = kBN * DK * 2;
   static constexpr int kVTileBytes = kBN * DV * 2;
   static constexpr int kStageBytes = kKTileBytes > kVTileBytes ? kKTileBytes : kVTileBytes;
-  static constexpr int kStages = QT == 1 ? (DK == 64 ? 5 : 2) : (DK == 64 && DV == 64) ? 8 : 4;
-  static constexpr int kOffQ = 0;
-  static constexpr int kOffKV = kOffQ + QT * kQTileBytes;
-  static constexpr int kOffBar = kOffKV + kStages * kStageBytes;
-  // P in TMEM columns of its own (d_v = 64: S0 S1 P0 P1 O0 O1 fill the 512 columns) lets the
-  // next block's scores be computed while the softmax still works on this block.  With
-  // d_v = 128 there is no room: P overwrites the S columns it came from.
+  // P in TMEM columns of its own (d_v = 64: S0 S1 P0 P1 O0 O1 fill the 512 columns), or in
+  // shared memory (d_v = 128: S0 S1 O0 O1 fill the TMEM, and P V becomes a shared-memory
+  // product).  Either way the next block's scores can be computed as soon as the softmax has
+  // read this block's S into registers.
   static constexpr bool kSepP = (DV == 64);
-  // With separate P, each Q tile gets its own issuing thread (its chain of products never
-  // waits behind the other tile's).  With P aliasing S, one thread issues both tiles' products
-  // back to back, which lets the first tile's scores finish early.
-  static constexpr int kIssuers = kSepP ? QT : 1;
+  static constexpr bool kSmemP = (DV == 128);
+  static constexpr int kPTileBytes = kSmemP ? kBM * kBN * 2 : 0;  // 128 rows x 128 keys bf16
+  static constexpr int kStages = QT == 1 ? (DK == 64 ? 5 : 2)
+                                 : (DK == 64 && DV == 64) ? 8
+                                 : kSmemP ? (DK == 128 ? 3 : 4) : 4;
+  static constexpr int kOffQ = 0;
+  static constexpr int kOffP = kOffQ + QT * kQTileBytes;
+  static constexpr int kOffKV = kOffP + QT * kPTileBytes;
+  static constexpr int kOffBar = kOffKV + kStages * kStageBytes;
+  // Each Q tile gets its own issuing thread (its chain of products never waits behind the
+  // other tile's).
+  static constexpr int kIssuers = QT;
   // barriers: full[NS], empty[NS], q_full, s_full[2], p_ready[2], o_done[2], s_free[2], p_free[2]
   static constexpr int kNumBars = 2 * kStages + 11;
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
@@ -173,6 +177,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   const uint32_t sQ = smem_u32(smem + C::kOffQ);
+  const uint32_t sP = smem_u32(smem + C::kOffP);
   const uint32_t sKV = smem_u32(smem + C::kOffKV);
   const uint32_t bar0 = smem_u32(smem + C::kOffBar);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
@@ -250,15 +255,12 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       uint32_t phase = 0;
       uint32_t issued = 0, issued_phase = 0;  // per slot: a load was issued / its phase bit
       bool aborted = false;
-      // Ring order = the MMA issuers' consumption order: K0 V0 K1 V1 ... (P aliasing S), or
-      // K0 K1 V0 K2 V1 ... (separate P: block n+1's scores come before block n's P V).
+      // Ring order = the MMA issuers' consumption order: K0 K1 V0 K2 V1 ... (block n+1's scores
+      // come before block n's P V).
       for (int t = 0; t < 2 * n_kt; ++t) {
         bool is_k;
         int n;
-        if (!C::kSepP) {
-          is_k = (t & 1) == 0;
-          n = t >> 1;
-        } else if (t == 0) {
+        if (t == 0) {
           is_k = true;
           n = 0;
         } else {
@@ -304,100 +306,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     // One issuing thread per Q tile, so that neither tile's products wait behind the other's.
     // Straight-line issue code: every operand of every tcgen05.mma is a loop invariant or an
     // unrolled constant offset, so each thread issues at the tensor pipe's rate.
-    if constexpr (!C::kSepP) {
-      if (lane == 0 && warp == kMmaWarp0) {
-        constexpr uint32_t kIdescQK = make_idesc(kBM, kBN, false);
-        constexpr uint32_t kIdescPV = make_idesc(kBM, DV, true);
-        const uint32_t tS0 = tmem + C::kTmemS0, tS1 = tmem + C::kTmemS1;
-        const uint32_t tO0 = tmem + C::kTmemO0, tO1 = tmem + C::kTmemO1;
-        const uint32_t sQ0 = sQ, sQ1 = sQ + C::kQTileBytes;
-        int slot = 0;
-        uint32_t phase = 0;
-        auto next = [&]() {
-          if (++slot == C::kStages) {
-            slot = 0;
-            phase ^= 1u;
-          }
-        };
-        // S = Q K^T: DK/16 MMAs (M=128, N=128, K=16), both operands K-major; the k-th step is
-        // panel k/4 of the 128-byte-swizzled tile, 32 bytes further for each step inside it.
-        auto issue_qk = [&](uint32_t tS, uint32_t qa, uint32_t kb) {
-#pragma unroll
-          for (int kk = 0; kk < DK / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * C::kPanelBytes + (kk & 3) * 32;
-            mma_f16_ss(tS, make_sdesc_sw128(qa + off, 16, 1024), make_sdesc_sw128(kb + off, 16, 1024),
-                       kIdescQK, kk > 0 ? 1u : 0u);
-          }
-        };
-        // O (+)= P V: 8 MMAs (M=128, N=DV, K=16).  A = P from TMEM (bf16 pairs: 8 columns per
-        // 16 keys).  B = V tile, MN-major: groups of 8 keys 1024 B apart (stride byte offset),
-        // 64-column panels kPanelBytes apart (leading byte offset).
-        auto issue_pv = [&](uint32_t tO, uint32_t tS, uint32_t vb, uint32_t acc_first) {
-#pragma unroll
-          for (int kk = 0; kk < kBN / 16; ++kk)
-            mma_f16_ts(tO, tS + kk * 8, make_sdesc_sw128(vb + kk * 2048, C::kPanelBytes, 1024),
-                       kIdescPV, kk > 0 ? 1u : acc_first);
-        };
-        bool ok = wait_bounded(q_full, 0, wc) && wait_bounded(full_bar(slot), phase, wc);
-        if (ok) {
-          tc_fence_after_sync();
-          const uint32_t kb = sKV + slot * C::kStageBytes;
-          const int ks = slot;
-          next();
-          issue_qk(tS0, sQ0, kb);
-          mma_commit(s_full(0));
-          issue_qk(tS1, sQ1, kb);
-          mma_commit(s_full(1));
-          mma_commit(empty_bar(ks));
-        }
-        for (int n = 1; ok && n < n_kt; ++n) {
-          const int vs = slot;
-          ok = wait_bounded(full_bar(slot), phase, wc);
-          next();
-          const int ks = slot;
-          ok = ok && wait_bounded(full_bar(slot), phase, wc);
-          next();
-          const uint32_t vb = sKV + vs * C::kStageBytes, kb = sKV + ks * C::kStageBytes;
-          const uint32_t par = uint32_t(n - 1) & 1u;
-          const uint32_t acc = n > 1 ? 1u : 0u;
-          ok = ok && wait_bounded(p_ready(0), par, wc);
-          if (!ok) break;
-          tc_fence_after_sync();
-          issue_pv(tO0, tS0, vb, acc);  // reads P0(n-1) before S0(n) overwrites those columns
-          issue_qk(tS0, sQ0, kb);
-          mma_commit(s_full(0));
-          ok = wait_bounded(p_ready(1), par, wc);
-          if (!ok) break;
-          tc_fence_after_sync();
-          issue_pv(tO1, tS1, vb, acc);
-          mma_commit(empty_bar(vs));
-          issue_qk(tS1, sQ1, kb);
-          mma_commit(s_full(1));
-          mma_commit(empty_bar(ks));
-        }
-        if (ok) {
-          const int vs = slot;
-          const uint32_t vb = sKV + vs * C::kStageBytes;
-          const uint32_t par = uint32_t(n_kt - 1) & 1u;
-          const uint32_t acc = n_kt > 1 ? 1u : 0u;
-          ok = wait_bounded(full_bar(slot), phase, wc) && wait_bounded(p_ready(0), par, wc);
-          if (ok) {
-            tc_fence_after_sync();
-            issue_pv(tO0, tS0, vb, acc);
-            ok = wait_bounded(p_ready(1), par, wc);
-          }
-          if (ok) {
-            tc_fence_after_sync();
-            issue_pv(tO1, tS1, vb, acc);
-            mma_commit(empty_bar(vs));
-          }
-        }
-        // Always signal the epilogue barrier once everything issued has completed, so that the
-        // TMEM is quiescent before it is freed even on the abort path.
-        mma_commit(o_done(0));
-        mma_commit(o_done(1));
-      }
-    } else if (lane == 0) {
+    if (lane == 0) {
       const int j = warp == kMmaWarp0 ? 0 : 1;
       constexpr uint32_t kIdescQK = make_idesc(kBM, kBN, false);
       constexpr uint32_t kIdescPV = make_idesc(kBM, DV, true);
@@ -405,6 +314,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       const uint32_t tP = tmem + (j ? C::kTmemP1 : C::kTmemP0);
       const uint32_t tO = tmem + (j ? C::kTmemO1 : C::kTmemO0);
       const uint32_t sQj = sQ + j * C::kQTileBytes;
+      const uint32_t sPj = sP + j * C::kPTileBytes;
       const uint32_t bar_s_full = s_full(j), bar_p_ready = p_ready(j), bar_s_free = s_free(j);
       const uint32_t bar_p_free = p_free(j);
       int slot = 0;
@@ -425,14 +335,22 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
                      make_sdesc_sw128(kb + off, 16, 1024), kIdescQK, kk > 0 ? 1u : 0u);
         }
       };
-      // O (+)= P V: 8 MMAs (M=128, N=DV, K=16).  A = P from TMEM (bf16 pairs: 8 columns per
-      // 16 keys).  B = V tile, MN-major: groups of 8 keys 1024 B apart (stride byte offset),
+      // O (+)= P V: 8 MMAs (M=128, N=DV, K=16).  A = P, from TMEM (bf16 pairs: 8 columns per
+      // 16 keys) or from shared memory (K-major, 128-byte swizzle, two 64-key panels: the layout
+      // of a Q tile).  B = V tile, MN-major: groups of 8 keys 1024 B apart (stride byte offset),
       // 64-column panels kPanelBytes apart (leading byte offset).
       auto issue_pv = [&](uint32_t vb, uint32_t acc_first) {
 #pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk)
-          mma_f16_ts(tO, tP + kk * 8, make_sdesc_sw128(vb + kk * 2048, C::kPanelBytes, 1024),
-                     kIdescPV, kk > 0 ? 1u : acc_first);
+        for (int kk = 0; kk < kBN / 16; ++kk) {
+          const uint64_t bdesc = make_sdesc_sw128(vb + kk * 2048, C::kPanelBytes, 1024);
+          if constexpr (C::kSmemP) {
+            const uint32_t off = (kk >> 2) * C::kPanelBytes + (kk & 3) * 32;
+            mma_f16_ss(tO, make_sdesc_sw128(sPj + off, 16, 1024), bdesc, kIdescPV,
+                       kk > 0 ? 1u : acc_first);
+          } else {
+            mma_f16_ts(tO, tP + kk * 8, bdesc, kIdescPV, kk > 0 ? 1u : acc_first);
+          }
+        }
       };
       bool ok = wait_bounded(q_full, 0, wc) && wait_bounded(full_bar(slot), phase, wc);
       // With d_k = 128, tile 1 starts once tile 0 holds its first scores in registers: the
@@ -448,7 +366,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         mma_commit(empty_bar(ks));
       }
       {
-        // P_j has columns of its own: S_j(n+1) is issued as soon as the softmax has read S_j(n),
+        // P_j has a buffer of its own: S_j(n+1) is issued as soon as the softmax has read S_j(n),
         // and O_j += P_j(n) V(n) once P_j(n) is written.
         for (int n = 0; ok && n < n_kt; ++n) {
           const uint32_t par = uint32_t(n) & 1u;
@@ -484,6 +402,10 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     const uint32_t tS = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemS1 : C::kTmemS0);
     const uint32_t tO = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemO1 : C::kTmemO0);
     const uint32_t tP = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemP1 : C::kTmemP0);
+    // This row of P_j in shared memory (d_v = 128): 16-byte chunk c of a 64-key panel sits at
+    // chunk c ^ (row & 7) of the row's 128 bytes (the 128-byte swizzle the MMA descriptor reads).
+    const uint32_t sProw = sP + j * C::kPTileBytes + uint32_t(row) * 128;
+    const uint32_t pswz = uint32_t(row & 7);
     const bool neg = c_log2 < 0.f;
     float m = -INFINITY;  // running maximum of c_log2 * s (log2 units)
     float l = 0.f;        // running sum of exp2(c_log2 * s - m)
@@ -496,11 +418,9 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       tc_fence_after_sync();
       uint32_t sr[128];
       tmem_load_row128(tS, sr);
-      if constexpr (C::kSepP) {
-        // S_j(n) is in registers: the MMA issuer may overwrite it with S_j(n+1).
-        tc_fence_before_sync();
-        mbar_arrive(s_free(j));
-      }
+      // S_j(n) is in registers: the MMA issuer may overwrite it with S_j(n+1).
+      tc_fence_before_sync();
+      mbar_arrive(s_free(j));
       float* s = reinterpret_cast<float*>(sr);
       // Keys of this tile that exist.
       const int valid = SPLIT ? min(kBN, *keys_from - n * kBN) : min(kBN, Nk - (kb0 + n) * kBN);
@@ -536,14 +456,12 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       const uint64_t mm = pack_f32x2(-m, -m);
       float l0 = 0.f, l1 = 0.f, l2 = 0.f, l3 = 0.f;
       const bool full = valid == kBN;
-      if constexpr (C::kSepP) {
-        // P_j's columns are free, and O_j may be rescaled, once O_j += P_j(n-1) V(n-1) is done.
-        if (n > 0 && !wait_bounded(p_free(j), uint32_t(n - 1) & 1u, wc)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after_sync();
+      // P_j's buffer is free, and O_j may be rescaled, once O_j += P_j(n-1) V(n-1) is done.
+      if (n > 0 && !wait_bounded(p_free(j), uint32_t(n - 1) & 1u, wc)) {
+        ok = false;
+        break;
       }
+      tc_fence_after_sync();
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         uint32_t pk[16];
@@ -566,13 +484,23 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           pk[i >> 1] = pack_bf16x2(p0, p1);
           pk[(i >> 1) + 1] = pack_bf16x2(p2, p3);
         }
-        tmem_st_32x32b_x16((C::kSepP ? tP : tS) + 16 * c, pk);
+        if constexpr (C::kSmemP) {
+          // keys 32c .. 32c+31: panel c/2, 16-byte chunks 4(c%2) .. 4(c%2)+3 of this row
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            st_shared_v4(sProw + (c >> 1) * C::kPanelBytes + ((uint32_t(4 * (c & 1) + i) ^ pswz) << 4),
+                         pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+        } else {
+          tmem_st_32x32b_x16(tP + 16 * c, pk);
+        }
       }
       l += (l0 + l1) + (l2 + l3);
       // O_j holds P V of tiles < n, complete because S_j(n) was committed after that product;
       // rescaled here, after the scores are dead, and before P_j(n) is released to the MMA.
       if (rescale) tmem_scale_row<DV>(tO, alpha);
       tmem_wait_st();
+      // P written by this thread in shared memory becomes visible to the tensor core's reads
+      if constexpr (C::kSmemP) fence_proxy_async_smem();
       tc_fence_before_sync();
       mbar_arrive(p_ready(j));
     }
