@@ -111,8 +111,14 @@ struct Cfg {
   // Each Q tile gets its own issuing thread (its chain of products never waits behind the
   // other tile's).
   static constexpr int kIssuers = QT;
-  // barriers: full[NS], empty[NS], q_full, s_full[2], p_ready[2], o_done[2], s_free[2], p_free[2]
-  static constexpr int kNumBars = 2 * kStages + 11;
+  // With P in shared memory (d_v = 128) the exponentials of the two Q tiles take turns: warp w
+  // of tile 0 and warp w + 4 of tile 1 share an SM sub-partition and its exp2 unit, and
+  // alternate their exponential phases (measured +1.4 % on 2x32x8192^2 and 1x16x32768^2, d=128;
+  // with d_v = 64 the same turns cost 8 % on 8x8x1024x4096).
+  static constexpr bool kTurns = QT == 2 && kSmemP;
+  // barriers: full[NS], empty[NS], q_full, s_full[2], p_ready[2], o_done[2], s_free[2],
+  // p_free[2], turn[4][2]
+  static constexpr int kNumBars = 2 * kStages + 11 + (kTurns ? 8 : 0);
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
   static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack for 1024-B alignment
   // Two tiles: S0 S1 P0 P1 O0 O1 (separate P) or S0 S1 O0 O1.  One tile: S0 P0 O0.
@@ -188,6 +194,8 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   auto o_done = [&](int j) { return bar0 + 8u * (2 * C::kStages + 5 + j); };
   auto s_free = [&](int j) { return bar0 + 8u * (2 * C::kStages + 7 + j); };
   auto p_free = [&](int j) { return bar0 + 8u * (2 * C::kStages + 9 + j); };
+  // turn(w, j): Q tile j's warp of lane quarter w may run its exponentials
+  auto turn = [&](int w, int j) { return bar0 + 8u * (2 * C::kStages + 11 + 2 * w + j); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
   // Split instance only: keys from this CTA's first key block to the end of the key axis, and
@@ -223,6 +231,11 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(s_free(j), 4 * 32);
       mbar_init(p_free(j), 1);
     }
+    if constexpr (C::kTurns)
+      for (int w = 0; w < 4; ++w) {
+        mbar_init(turn(w, 0), 1);
+        mbar_init(turn(w, 1), 1);
+      }
     *abort_flag = 0;
     if constexpr (SPLIT) {
       *keys_from = Nk - kb0 * kBN;
@@ -410,6 +423,11 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     float m = -INFINITY;  // running maximum of c_log2 * s (log2 units)
     float l = 0.f;        // running sum of exp2(c_log2 * s - m)
     bool ok = true;
+    // Exponential turns: tile 0 goes first in every key block.  turn(w, 0) completes its phase
+    // n when tile 1's warp has finished block n - 1 (phase 0: at the start), turn(w, 1) its
+    // phase n when tile 0's warp has finished block n; neither can run two phases ahead.
+    const int quarter = warp & 3;
+    if (C::kTurns && j == 1 && lane == 0) mbar_arrive(turn(quarter, 0));
     for (int n = 0; n < n_kt; ++n) {
       if (!wait_bounded(s_full(j), uint32_t(n) & 1u, wc)) {
         ok = false;
@@ -462,6 +480,10 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         break;
       }
       tc_fence_after_sync();
+      if (C::kTurns && !wait_bounded(turn(quarter, j), uint32_t(n) & 1u, wc)) {
+        ok = false;
+        break;
+      }
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         uint32_t pk[16];
@@ -493,6 +515,10 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         } else {
           tmem_st_32x32b_x16(tP + 16 * c, pk);
         }
+      }
+      if constexpr (C::kTurns) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(turn(quarter, j ^ 1));
       }
       l += (l0 + l1) + (l2 + l3);
       // O_j holds P V of tiles < n, complete because S_j(n) was committed after that product;
