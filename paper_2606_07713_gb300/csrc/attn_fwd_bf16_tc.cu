@@ -67,17 +67,17 @@ constexpr int kBM = 128;          // query rows per Q tile (= TMEM lanes)
 constexpr int kBN = 128;          // keys per K/V tile
 constexpr int kQTiles = 2;        // Q tiles per CTA of the two-tile kernel
 constexpr float kRescaleLog2 = 8.0f;  // lazy-rescale threshold: exponentials stay <= 2^8
-// Longest suspension of one mbarrier test for the two-tile d_v = 64 schedule, where the MMA
-// and TMA threads wait long enough that polling would take issue slots from the softmax warps
-// (measured +3.6% there, -1..3% with d_v = 128, which therefore polls).  One-tile CTAs poll:
-// with the suspension they ran at 709 TFLOP/s instead of 740 on 4x16x2048^2.
+// Longest suspension of one mbarrier test in the two-tile kernel, where the MMA and TMA threads
+// wait long enough that polling would take issue slots from the softmax warps (measured +3.6 %
+// with d_v = 64).  One-tile CTAs poll: with the suspension they ran at 709 TFLOP/s instead of
+// 740 on 4x16x2048^2.
 constexpr uint32_t kWaitHintNs = 20000;
 
 template <int DK, int DV, int QT = 2>
 struct Cfg {
   static_assert(DK == 64 || DK == 128, "d_k must be 64 or 128");
   static_assert(QT == 1 || QT == 2, "one or two Q tiles per CTA");
-  static_assert(QT == 2 || DV == 64, "one-tile CTAs use the separate-P schedule");
+  static_assert(QT == 2 || DV == 64, "one-tile CTAs hold S, P and O of d_v = 64");
   // Warps: 4 softmax warps per Q tile, then the MMA warp of tile 0 (it also allocates and frees
   // TMEM), the TMA warp and, with two tiles, the MMA warp of tile 1.  One-tile CTAs run two per
   // SM (half the registers, TMEM and shared memory each).
@@ -94,38 +94,37 @@ struct Cfg {
   static constexpr int kKTileBytes = kBN * DK * 2;
   static constexpr int kVTileBytes = kBN * DV * 2;
   static constexpr int kStageBytes = kKTileBytes > kVTileBytes ? kKTileBytes : kVTileBytes;
-  // P in TMEM columns of its own (d_v = 64: S0 S1 P0 P1 O0 O1 fill the 512 columns), or in
-  // shared memory (d_v = 128: S0 S1 O0 O1 fill the TMEM, and P V becomes a shared-memory
-  // product).  Either way the next block's scores can be computed as soon as the softmax has
-  // read this block's S into registers.
-  static constexpr bool kSepP = (DV == 64);
-  static constexpr bool kSmemP = (DV == 128);
-  static constexpr int kPTileBytes = kSmemP ? kBM * kBN * 2 : 0;  // 128 rows x 128 keys bf16
+  // P has TMEM columns of its own, so the next block's scores can be computed as soon as the
+  // softmax has read this block's S into registers.  Two tiles with d_v = 64: S0 S1 P0 P1 O0 O1
+  // fill the 512 columns.  Two tiles with d_v = 128: O0 O1 take 256 columns, so the two tiles
+  // share one S buffer (S P0 P1 O0 O1), and their score products alternate: tile 1's S(n) is
+  // computed once tile 0's softmax holds S(n) in registers, tile 0's S(n+1) once tile 1's
+  // softmax holds its S(n).  (P in shared memory instead, with an S buffer per tile, measured
+  // the same; it moves 128 KB more per key block through shared memory.)  One tile: S0 P0 O0.
+  static constexpr bool kSharedS = QT == 2 && DV == 128;
   static constexpr int kStages = QT == 1 ? (DK == 64 ? 5 : 2)
                                  : (DK == 64 && DV == 64) ? 8
-                                 : kSmemP ? (DK == 128 ? 3 : 4) : 4;
+                                 : kSharedS ? (DK == 128 ? 5 : 6) : 4;
   static constexpr int kOffQ = 0;
-  static constexpr int kOffP = kOffQ + QT * kQTileBytes;
-  static constexpr int kOffKV = kOffP + QT * kPTileBytes;
+  static constexpr int kOffKV = kOffQ + QT * kQTileBytes;
   static constexpr int kOffBar = kOffKV + kStages * kStageBytes;
   // Each Q tile gets its own issuing thread (its chain of products never waits behind the
   // other tile's).
   static constexpr int kIssuers = QT;
-  // With P in shared memory (d_v = 128) the exponentials of the two Q tiles take turns: warp w
-  // of tile 0 and warp w + 4 of tile 1 share an SM sub-partition and its exp2 unit, and
-  // alternate their exponential phases (measured +1.4 % on 2x32x8192^2 and 1x16x32768^2, d=128;
-  // with d_v = 64 the same turns cost 8 % on 8x8x1024x4096).
-  static constexpr bool kTurns = QT == 2 && kSmemP;
-  // barriers: full[NS], empty[NS], q_full, s_full[2], p_ready[2], o_done[2], s_free[2],
-  // p_free[2], turn[4][2]
-  static constexpr int kNumBars = 2 * kStages + 11 + (kTurns ? 8 : 0);
+  // Chunks of 32 exponentials computed before the wait for P's buffer (the rest after it), so
+  // that the wait for the previous block's P V overlaps them (measured on 4x16x2048^2, d=64:
+  // 0 -> 2 chunks 740 -> 812 TFLOP/s; 1x16x32768^2, d=128: 0 -> 3 chunks +2 %; more chunks
+  // spill registers and run slower).
+  static constexpr int kEarlyChunks = QT == 1 ? 2 : DV == 64 ? 0 : 3;
+  // barriers: full[NS], empty[NS], q_full, s_full[2], p_ready[2], o_done[2], s_free[2], p_free[2]
+  static constexpr int kNumBars = 2 * kStages + 11;
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
   static constexpr int kSmemBytes = kOffMisc + 16 + 1024;  // + slack for 1024-B alignment
-  // Two tiles: S0 S1 P0 P1 O0 O1 (separate P) or S0 S1 O0 O1.  One tile: S0 P0 O0.
-  static constexpr uint32_t kTmemS0 = 0, kTmemS1 = 128;
-  static constexpr uint32_t kTmemP0 = kSepP ? 128 * QT : kTmemS0;
-  static constexpr uint32_t kTmemP1 = kSepP ? 320 : kTmemS1;
-  static constexpr uint32_t kTmemO0 = kSepP ? 192 * QT : 256, kTmemO1 = kTmemO0 + DV;
+  static constexpr uint32_t kTmemS0 = 0, kTmemS1 = kSharedS ? 0 : 128;
+  static constexpr uint32_t kTmemP0 = kSharedS ? 128 : 128 * QT;
+  static constexpr uint32_t kTmemP1 = kSharedS ? 192 : 320;
+  static constexpr uint32_t kTmemO0 = kSharedS ? 256 : 192 * QT;
+  static constexpr uint32_t kTmemO1 = kTmemO0 + DV;
   static_assert((QT == 2 ? kTmemO1 : kTmemO0) + DV <= kTmemCols, "TMEM budget");
   // Per SM: 228 KB, 1 KB of it reserved per CTA.
   static_assert(kSmemBytes <= (QT == 2 ? 232448 : 233472 / 2 - 1024), "shared memory budget");
@@ -183,7 +182,6 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   const uint32_t sQ = smem_u32(smem + C::kOffQ);
-  const uint32_t sP = smem_u32(smem + C::kOffP);
   const uint32_t sKV = smem_u32(smem + C::kOffKV);
   const uint32_t bar0 = smem_u32(smem + C::kOffBar);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
@@ -194,8 +192,6 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   auto o_done = [&](int j) { return bar0 + 8u * (2 * C::kStages + 5 + j); };
   auto s_free = [&](int j) { return bar0 + 8u * (2 * C::kStages + 7 + j); };
   auto p_free = [&](int j) { return bar0 + 8u * (2 * C::kStages + 9 + j); };
-  // turn(w, j): Q tile j's warp of lane quarter w may run its exponentials
-  auto turn = [&](int w, int j) { return bar0 + 8u * (2 * C::kStages + 11 + 2 * w + j); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kOffMisc + 4);
   // Split instance only: keys from this CTA's first key block to the end of the key axis, and
@@ -215,7 +211,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   // This CTA's key blocks: [kb0, kb0 + n_kt) (all of them unless the key axis is split).
   const int kb0 = SPLIT ? split * kv_per_split : 0;
   const int n_kt = SPLIT ? min((Nk + kBN - 1) / kBN - kb0, kv_per_split) : (Nk + kBN - 1) / kBN;
-  const WaitCtl wc{abort_flag, wait_limit_ns, C::kSepP && QT == 2 ? kWaitHintNs : 0u,
+  const WaitCtl wc{abort_flag, wait_limit_ns, QT == 2 ? kWaitHintNs : 0u,
                    &g_moa_bf16_status};
 
   if (threadIdx.x == 0) {
@@ -231,11 +227,6 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(s_free(j), 4 * 32);
       mbar_init(p_free(j), 1);
     }
-    if constexpr (C::kTurns)
-      for (int w = 0; w < 4; ++w) {
-        mbar_init(turn(w, 0), 1);
-        mbar_init(turn(w, 1), 1);
-      }
     *abort_flag = 0;
     if constexpr (SPLIT) {
       *keys_from = Nk - kb0 * kBN;
@@ -327,7 +318,6 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       const uint32_t tP = tmem + (j ? C::kTmemP1 : C::kTmemP0);
       const uint32_t tO = tmem + (j ? C::kTmemO1 : C::kTmemO0);
       const uint32_t sQj = sQ + j * C::kQTileBytes;
-      const uint32_t sPj = sP + j * C::kPTileBytes;
       const uint32_t bar_s_full = s_full(j), bar_p_ready = p_ready(j), bar_s_free = s_free(j);
       const uint32_t bar_p_free = p_free(j);
       int slot = 0;
@@ -348,28 +338,20 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
                      make_sdesc_sw128(kb + off, 16, 1024), kIdescQK, kk > 0 ? 1u : 0u);
         }
       };
-      // O (+)= P V: 8 MMAs (M=128, N=DV, K=16).  A = P, from TMEM (bf16 pairs: 8 columns per
-      // 16 keys) or from shared memory (K-major, 128-byte swizzle, two 64-key panels: the layout
-      // of a Q tile).  B = V tile, MN-major: groups of 8 keys 1024 B apart (stride byte offset),
+      // O (+)= P V: 8 MMAs (M=128, N=DV, K=16).  A = P from TMEM (bf16 pairs: 8 columns per
+      // 16 keys).  B = V tile, MN-major: groups of 8 keys 1024 B apart (stride byte offset),
       // 64-column panels kPanelBytes apart (leading byte offset).
       auto issue_pv = [&](uint32_t vb, uint32_t acc_first) {
 #pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk) {
-          const uint64_t bdesc = make_sdesc_sw128(vb + kk * 2048, C::kPanelBytes, 1024);
-          if constexpr (C::kSmemP) {
-            const uint32_t off = (kk >> 2) * C::kPanelBytes + (kk & 3) * 32;
-            mma_f16_ss(tO, make_sdesc_sw128(sPj + off, 16, 1024), bdesc, kIdescPV,
-                       kk > 0 ? 1u : acc_first);
-          } else {
-            mma_f16_ts(tO, tP + kk * 8, bdesc, kIdescPV, kk > 0 ? 1u : acc_first);
-          }
-        }
+        for (int kk = 0; kk < kBN / 16; ++kk)
+          mma_f16_ts(tO, tP + kk * 8, make_sdesc_sw128(vb + kk * 2048, C::kPanelBytes, 1024),
+                     kIdescPV, kk > 0 ? 1u : acc_first);
       };
       bool ok = wait_bounded(q_full, 0, wc) && wait_bounded(full_bar(slot), phase, wc);
       // With d_k = 128, tile 1 starts once tile 0 holds its first scores in registers: the
       // tiles' reads of S from tensor memory then stop coinciding (measured +2 % on
       // 8x8x1024x4096, d_k = 128, d_v = 64; -2 % with d_k = 64, which therefore starts both).
-      if (DK == 128 && j == 1) ok = ok && wait_bounded(s_free(0), 0, wc);
+      if ((DK == 128 || C::kSharedS) && j == 1) ok = ok && wait_bounded(s_free(0), 0, wc);
       if (ok) {
         tc_fence_after_sync();
         const int ks = slot;
@@ -385,7 +367,12 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           const uint32_t par = uint32_t(n) & 1u;
           if (n + 1 < n_kt) {
             const int ks = slot;
-            ok = wait_bounded(full_bar(slot), phase, wc) && wait_bounded(bar_s_free, par, wc);
+            // The S buffer may take block n+1's scores once its last reader has them in
+            // registers: this tile's softmax (own S buffer), or with one S buffer shared by the
+            // two tiles, the other tile's softmax (block n for tile 0, block n+1 for tile 1).
+            ok = wait_bounded(full_bar(slot), phase, wc) &&
+                 (C::kSharedS ? wait_bounded(s_free(j ^ 1), j ? (par ^ 1u) : par, wc)
+                              : wait_bounded(bar_s_free, par, wc));
             next();
             if (!ok) break;
             tc_fence_after_sync();
@@ -415,19 +402,10 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
     const uint32_t tS = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemS1 : C::kTmemS0);
     const uint32_t tO = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemO1 : C::kTmemO0);
     const uint32_t tP = tmem + (uint32_t(lane_base) << 16) + (j ? C::kTmemP1 : C::kTmemP0);
-    // This row of P_j in shared memory (d_v = 128): 16-byte chunk c of a 64-key panel sits at
-    // chunk c ^ (row & 7) of the row's 128 bytes (the 128-byte swizzle the MMA descriptor reads).
-    const uint32_t sProw = sP + j * C::kPTileBytes + uint32_t(row) * 128;
-    const uint32_t pswz = uint32_t(row & 7);
     const bool neg = c_log2 < 0.f;
     float m = -INFINITY;  // running maximum of c_log2 * s (log2 units)
     float l = 0.f;        // running sum of exp2(c_log2 * s - m)
     bool ok = true;
-    // Exponential turns: tile 0 goes first in every key block.  turn(w, 0) completes its phase
-    // n when tile 1's warp has finished block n - 1 (phase 0: at the start), turn(w, 1) its
-    // phase n when tile 0's warp has finished block n; neither can run two phases ahead.
-    const int quarter = warp & 3;
-    if (C::kTurns && j == 1 && lane == 0) mbar_arrive(turn(quarter, 0));
     for (int n = 0; n < n_kt; ++n) {
       if (!wait_bounded(s_full(j), uint32_t(n) & 1u, wc)) {
         ok = false;
@@ -474,19 +452,8 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       const uint64_t mm = pack_f32x2(-m, -m);
       float l0 = 0.f, l1 = 0.f, l2 = 0.f, l3 = 0.f;
       const bool full = valid == kBN;
-      // P_j's buffer is free, and O_j may be rescaled, once O_j += P_j(n-1) V(n-1) is done.
-      if (n > 0 && !wait_bounded(p_free(j), uint32_t(n - 1) & 1u, wc)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after_sync();
-      if (C::kTurns && !wait_bounded(turn(quarter, j), uint32_t(n) & 1u, wc)) {
-        ok = false;
-        break;
-      }
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t pk[16];
+      // Chunk c of 32 scores -> p = exp2(c*s - m), row sums, bf16 pairs in pk.
+      auto exp_chunk = [&](int c, uint32_t* pk) {
 #pragma unroll
         for (int i = 0; i < 32; i += 4) {
           const int k = 32 * c + i;
@@ -506,27 +473,34 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           pk[i >> 1] = pack_bf16x2(p0, p1);
           pk[(i >> 1) + 1] = pack_bf16x2(p2, p3);
         }
-        if constexpr (C::kSmemP) {
-          // keys 32c .. 32c+31: panel c/2, 16-byte chunks 4(c%2) .. 4(c%2)+3 of this row
+      };
+      // Chunk c of P to where O += P V reads it: 16 packed TMEM columns at column 16c.
+      auto store_chunk = [&](int c, const uint32_t* pk) { tmem_st_32x32b_x16(tP + 16 * c, pk); };
+      // The first kEarlyChunks chunks are computed before waiting for P_j's buffer, so that
+      // the wait overlaps their exponentials.
+      constexpr int kEarly = C::kEarlyChunks;
+      uint32_t pe[kEarly > 0 ? 16 * kEarly : 1];
 #pragma unroll
-          for (int i = 0; i < 4; ++i)
-            st_shared_v4(sProw + (c >> 1) * C::kPanelBytes + ((uint32_t(4 * (c & 1) + i) ^ pswz) << 4),
-                         pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
-        } else {
-          tmem_st_32x32b_x16(tP + 16 * c, pk);
-        }
+      for (int c = 0; c < kEarly; ++c) exp_chunk(c, pe + 16 * c);
+      // P_j's buffer is free, and O_j may be rescaled, once O_j += P_j(n-1) V(n-1) is done.
+      if (n > 0 && !wait_bounded(p_free(j), uint32_t(n - 1) & 1u, wc)) {
+        ok = false;
+        break;
       }
-      if constexpr (C::kTurns) {
-        __syncwarp();
-        if (lane == 0) mbar_arrive(turn(quarter, j ^ 1));
+      tc_fence_after_sync();
+#pragma unroll
+      for (int c = 0; c < kEarly; ++c) store_chunk(c, pe + 16 * c);
+#pragma unroll
+      for (int c = kEarly; c < 4; ++c) {
+        uint32_t pk[16];
+        exp_chunk(c, pk);
+        store_chunk(c, pk);
       }
       l += (l0 + l1) + (l2 + l3);
       // O_j holds P V of tiles < n, complete because S_j(n) was committed after that product;
       // rescaled here, after the scores are dead, and before P_j(n) is released to the MMA.
       if (rescale) tmem_scale_row<DV>(tO, alpha);
       tmem_wait_st();
-      // P written by this thread in shared memory becomes visible to the tensor core's reads
-      if constexpr (C::kSmemP) fence_proxy_async_smem();
       tc_fence_before_sync();
       mbar_arrive(p_ready(j));
     }

@@ -65,14 +65,6 @@ __device__ __forceinline__ bool mbar_try_wait_hint(uint32_t bar, uint32_t parity
   return ok != 0;
 }
 
-// 16-byte store to shared memory (a 32-bit shared-window address).
-__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
-                                             uint32_t d) {
-  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
-               "r"(d)
-               : "memory");
-}
-
 // ---------------------------------------------------------------------------------------------
 // TMA (cp.async.bulk.tensor), 3-D tiled copies global -> shared, completion on an mbarrier
 // ---------------------------------------------------------------------------------------------
