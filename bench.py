@@ -8,7 +8,7 @@ launch).  `--workload 2` selects the small d=64 case, 3 and 4 the other bf16 sha
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference|classical]
                     [--workload ID] [--shape B,H,N_q,N_k,d_k,d_v] [--pass fwd|bwd|qkv]
-                    [--shard bh|replica]
+                    [--scaling weak|strong]
 
 Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s: FLOPs of every step on every
 rank divided by the slowest rank's summed kernel time, measured with CUDA events on the
@@ -24,15 +24,18 @@ times moa_attn_bwd (three launches) on the same workload instead of the forward 
 `--pass qkv` the fused projection moa_qkv_proj producing that workload's Q, K, V from an input
 X [B, N, H*d_k].
 
-Multi-GPU (torchrun), forward pass: by default (`--shard bh`) the workload's B*H independent
-(b, h) slices are partitioned into contiguous ranges, one per rank, and each rank runs the
-forward on its own range only: no collective touches the data (one all_reduce(MAX) of the
-timings), and the total work is fixed, so scaling is strong.  `--shard replica` instead runs the
-whole workload on every rank (weak scaling); the backward and projection passes always do that.
+Multi-GPU (torchrun), forward pass: the (b, h) slices of the job are independent problems and
+are partitioned into contiguous ranges, one per rank; each rank runs the forward on its own
+range only, and no collective touches the data (one all_reduce(MAX) of the timings).  By default
+(`--scaling weak`) the job on N GPUs is N seeded instances of the workload, N*B*H slices, so
+every rank owns B*H of them (rank r: the instance with seed s + 1000 r).  `--scaling strong`
+partitions the workload's own B*H slices instead (fixed total work).  The backward and
+projection passes run the whole workload on every rank.
 """
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import math
@@ -221,6 +224,19 @@ def job_tflops(job_flops_per_step: float, steps: int, max_ms: float) -> float:
     return job_flops_per_step * steps / (max_ms * 1e-3) / 1e12
 
 
+def rank_slices(scaling: str, bh: int, world: int, rank: int, seed: int):
+    """(lo, hi, job_slices, seed) of this rank's part of the forward job.  The job's (b, h) slices
+    are partitioned into contiguous ranges (shard.bh_range).  Weak scaling: the job is `world`
+    seeded instances of the workload (world * bh slices), so rank r owns exactly instance r,
+    drawn with seed + 1000 r.  Strong scaling: the job is the workload's own bh slices, split."""
+    from paper_2606_07713_gb300 import shard as SH
+    if scaling == "strong":
+        lo, hi = SH.bh_range(bh, world, rank)
+        return lo, hi, bh, seed
+    lo, hi = SH.bh_range(world * bh, world, rank)
+    return lo, hi, world * bh, seed + 1000 * rank
+
+
 def to_device_bf16(bits, dev):
     import torch
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
@@ -256,15 +272,16 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
     torch.cuda.set_device(dev)
     pkg.lib()
     s = cfg.shape
-    x = I.make_inputs(cfg)
-    # This rank's (b, h) slices: a contiguous range of the flattened B*H axis (--shard bh), or
-    # all of them (one GPU, or --shard replica).  A range is one contiguous block of each tensor.
+    # This rank's (b, h) slices: a contiguous range of the job's slices (rank_slices).  A range
+    # is one contiguous block of each tensor of its workload instance.
     bh_total = s.B * s.H
-    sharded = world > 1 and args.shard == "bh"
-    lo, hi = SH.bh_range(bh_total, world, rank) if sharded else (0, bh_total)
+    strong = world > 1 and args.scaling == "strong"
+    lo, hi, job_slices, seed = rank_slices(args.scaling, bh_total, world, rank, cfg.the_seed)
+    x = I.make_inputs(cfg if seed == cfg.the_seed else dataclasses.replace(cfg, seed=seed))
     n_sl = hi - lo
 
-    hb = [SH.block(a, lo, hi) for a in ((x.q_bits, x.k_bits, x.v_bits) if cfg.dtype == "bf16"
+    lo_i, hi_i = (lo, hi) if strong else (0, bh_total)   # the range inside this rank's instance
+    hb = [SH.block(a, lo_i, hi_i) for a in ((x.q_bits, x.k_bits, x.v_bits) if cfg.dtype == "bf16"
                                          else (x.q, x.k, x.v))]
     if cfg.dtype == "bf16":
         hq, hk, hv = (torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).pin_memory() for b in hb)
@@ -278,7 +295,7 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
     code = pkg.MOA_BF16 if cfg.dtype == "bf16" else pkg.MOA_FP32
     rank_flops = pkg.attn_flops(1, n_sl, s.N_q, s.N_k, s.d_k, s.d_v) if n_sl else 0.0
     flops = pkg.attn_flops(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v)
-    job_flops = flops if sharded else flops * world
+    job_flops = flops * job_slices / bh_total
     dnf = pkg.dnf_bytes(s.B, s.H, s.N_q, s.N_k, s.d_k, s.d_v, code)
     elt = 2 if cfg.dtype == "bf16" else 4
 
@@ -351,7 +368,7 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
                             elt * bh_total * s.N_q * s.d_v)
         in_bytes = elt * bh_total * (s.N_q * s.d_k + s.N_k * s.d_k + s.N_k * s.d_v)
         out_bytes = elt * bh_total * s.N_q * s.d_v
-        copies = 1 if sharded else world
+        copies = job_slices / bh_total
         line = {
             "metric": METRIC,
             "value": round(value, 2),
@@ -361,14 +378,15 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
             "warmup": args.warmup,
             "ms_per_step": round(total_ms / args.steps, 6),
             "higher_is_better": True,
-            "scaling": "strong" if sharded else "weak",
+            "scaling": "strong" if strong else "weak",
             "vs_baseline": None,
             "dtype": cfg.dtype,
             "data": "synthetic: seeded splitmix64 + Box-Muller inputs of the workload's shape",
             "config": dict(workload_desc(cfg), parallelism=(
-                f"B*H slices partitioned over {world} ranks (contiguous ranges, no data "
-                f"collective)" if sharded else
-                ("one GPU" if world == 1 else f"{world} replicas of the whole workload"))),
+                "one GPU" if world == 1 else
+                f"{job_slices} (b, h) slices partitioned over {world} ranks in contiguous ranges "
+                f"({'the workload split' if strong else 'one seeded workload instance per rank'}; "
+                f"no data collective)")),
             "pct_of_bf16_peak": round(100.0 * achieved / float(peaks["bf16_tflops"]), 2),
             "dnf_bytes": dnf,
             "roofline": {
@@ -394,7 +412,7 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
                 "api": "moa_attn_fwd_staged",
             },
             # one kernel per step on every rank that owns at least one slice
-            "gpu_launches": args.steps * (min(world, bh_total) if sharded else world),
+            "gpu_launches": args.steps * min(world, job_slices),
             "clocks": clocks,
             "wall_s_timed_loop": round(wall, 4),
         }
@@ -897,9 +915,10 @@ def main():
                     help="backward kernels: fused (one tile kernel, d_k = d_v = 64; its dQ is not "
                          "bitwise reproducible), split (dK/dV and dQ kernels; bitwise "
                          "reproducible), auto (fused where it applies)")
-    ap.add_argument("--shard", choices=["bh", "replica"], default="bh",
-                    help="forward pass on N > 1 GPUs: bh partitions the B*H slices over the ranks "
-                         "(strong scaling), replica runs the whole workload on every rank (weak)")
+    ap.add_argument("--scaling", choices=["weak", "strong"], default="weak",
+                    help="forward pass on N > 1 GPUs, slices partitioned over the ranks: weak = a "
+                         "job of N workload instances (B*H slices per rank), strong = the "
+                         "workload's own B*H slices split")
     ap.add_argument("--pass", dest="which", choices=["fwd", "bwd", "qkv"], default="fwd",
                     help="time the forward (default), the backward pass or the QKV projection")
     ap.add_argument("--shape", default=None,

@@ -71,3 +71,19 @@ def test_job_value_strong_and_weak():
     # strong: the job's FLOPs are fixed; weak (replicas): they grow with the rank count
     assert bench.job_tflops(1e12, 10, 1000.0) == pytest.approx(10.0)
     assert bench.whole_job_tflops(1e12, 10, 4, 1000.0) == pytest.approx(40.0)
+
+
+def test_rank_slices_weak_and_strong():
+    from paper_2606_07713_gb300 import shard as SH
+    # weak: rank r owns instance r of the job (its own seed), bh slices each
+    for world in (1, 2, 3, 8):
+        got = [bench.rank_slices("weak", 16, world, r, 5) for r in range(world)]
+        assert [(lo, hi) for lo, hi, _, _ in got] == [(16 * r, 16 * (r + 1)) for r in range(world)]
+        assert all(js == 16 * world for _, _, js, _ in got)
+        assert [sd for _, _, _, sd in got] == [5 + 1000 * r for r in range(world)]
+    # strong: the workload's own slices split; every rank keeps the workload's seed
+    got = [bench.rank_slices("strong", 14, 4, r, 3) for r in range(4)]
+    assert [(lo, hi) for lo, hi, _, _ in got] == SH.bh_ranges(14, 4)
+    assert all(js == 14 and sd == 3 for _, _, js, sd in got)
+    # one GPU: both modes are the whole workload
+    assert bench.rank_slices("weak", 16, 1, 0, 5) == bench.rank_slices("strong", 16, 1, 0, 5) == (0, 16, 16, 5)
