@@ -86,9 +86,14 @@ def measured_peaks() -> tuple[dict, str]:
 
 
 def kernel_source_hash() -> str:
+    """sha256 of the forward kernel's sources with comments and whitespace removed, so that an
+    ncu summary stays tied to the code it measured and not to its comments."""
     h = hashlib.sha256()
     for f in KERNEL_SOURCES:
-        h.update(open(f, "rb").read())
+        text = open(f).read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        h.update(" ".join(text.split()).encode())
     return h.hexdigest()
 
 

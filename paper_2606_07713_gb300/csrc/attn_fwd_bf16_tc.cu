@@ -348,8 +348,9 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
                      kIdescPV, kk > 0 ? 1u : acc_first);
       };
       bool ok = wait_bounded(q_full, 0, wc) && wait_bounded(full_bar(slot), phase, wc);
-      // With d_k = 128, tile 1 starts once tile 0 holds its first scores in registers: the
-      // tiles' reads of S from tensor memory then stop coinciding (measured +2 % on
+      // Tile 1's first scores wait until tile 0 holds its own in registers: required with one
+      // S buffer for both tiles (d_v = 128); with an S buffer per tile and d_k = 128 it keeps
+      // the tiles' reads of S from tensor memory from coinciding (measured +2 % on
       // 8x8x1024x4096, d_k = 128, d_v = 64; -2 % with d_k = 64, which therefore starts both).
       if ((DK == 128 || C::kSharedS) && j == 1) ok = ok && wait_bounded(s_free(0), 0, wc);
       if (ok) {
@@ -361,8 +362,8 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
         mma_commit(empty_bar(ks));
       }
       {
-        // P_j has a buffer of its own: S_j(n+1) is issued as soon as the softmax has read S_j(n),
-        // and O_j += P_j(n) V(n) once P_j(n) is written.
+        // P_j has TMEM columns of its own: S_j(n+1) is issued as soon as the S buffer's last
+        // reader has its scores in registers, and O_j += P_j(n) V(n) once P_j(n) is written.
         for (int n = 0; ok && n < n_kt; ++n) {
           const uint32_t par = uint32_t(n) & 1u;
           if (n + 1 < n_kt) {
