@@ -67,12 +67,10 @@ constexpr int kBM = 128;          // query rows per Q tile (= TMEM lanes)
 constexpr int kBN = 128;          // keys per K/V tile
 constexpr int kQTiles = 2;        // Q tiles per CTA of the two-tile kernel
 constexpr float kRescaleLog2 = 8.0f;  // lazy-rescale threshold: exponentials stay <= 2^8
-// Longest suspension of one mbarrier test in the two-tile d_v = 64 kernel, where the MMA and TMA
-// threads wait long enough that polling would take issue slots from the softmax warps (measured
-// +3.6 %).  The other kernels poll: the one-tile kernel ran at 709 TFLOP/s with the suspension
-// instead of 740 on 4x16x2048^2, and the d_v = 128 kernel (one S buffer) at 1638 / 1656 instead
-// of 1712 / 1712 on 2x32x8192^2 / 1x16x32768^2.
-constexpr uint32_t kWaitHintNs = 20000;
+// Every wait polls.  A suspension hint on the MMA issuers' and TMA producer's waits (20 us) gave
+// +3.6 % with an earlier d_v = 64 schedule; with the current schedules it is neutral there and
+// costs 4 % at d_v = 128 (1712 -> 1638 TFLOP/s on 2x32x8192^2), where the MMA issuers' waits are
+// on the critical path; the one-tile kernel ran at 709 instead of 740 with it.
 
 template <int DK, int DV, int QT = 2>
 struct Cfg {
@@ -212,8 +210,7 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   // This CTA's key blocks: [kb0, kb0 + n_kt) (all of them unless the key axis is split).
   const int kb0 = SPLIT ? split * kv_per_split : 0;
   const int n_kt = SPLIT ? min((Nk + kBN - 1) / kBN - kb0, kv_per_split) : (Nk + kBN - 1) / kBN;
-  const WaitCtl wc{abort_flag, wait_limit_ns, (QT == 2 && DV == 64) ? kWaitHintNs : 0u,
-                   &g_moa_bf16_status};
+  const WaitCtl wc{abort_flag, wait_limit_ns, 0u, &g_moa_bf16_status};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
