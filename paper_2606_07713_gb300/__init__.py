@@ -175,10 +175,12 @@ def qkv_proj(x, w, H: int, d_k: int, d_v: int, out=None, stream=None):
 
 def attn_fwd_splitkv(q, k, v, num_splits: int = MOA_SPLITS_AUTO, scale: float | None = None,
                      out=None, workspace=None, stream=None):
-    """attn_fwd with the key axis split into up to num_splits ranges merged at the end; with
-    MOA_SPLITS_AUTO (0) only the query blocks of the last partial wave are split, as the library
-    chooses for q's device.  The workspace (a CUDA uint8 tensor of at least
-    moa_attn_splitkv_workspace_bytes(...) bytes) is allocated here when not given."""
+    """attn_fwd with the key axis split into up to num_splits ranges merged at the end.  With
+    MOA_SPLITS_AUTO (0) the library chooses from q's device: when the 256-row query blocks leave
+    SMs idle, every block's key axis is split so that the CTAs fill the SMs (if its cost model
+    predicts a saving); otherwise nothing is split and the result is attn_fwd's.  The workspace
+    (a CUDA uint8 tensor of at least moa_attn_splitkv_workspace_bytes(...) bytes) is allocated
+    here when not given."""
     import torch
     for t in (q, k, v):
         if not t.is_cuda or not t.is_contiguous():
