@@ -20,9 +20,8 @@ M_classical models (Section 8.2): the score matrix, its max-shifted exponentials
 normalised weights each materialised in device memory by eager PyTorch ops (cuBLAS GEMMs and
 elementwise/reduction kernels) -- a measurement of the comparison, not part of the library.
 `--shape` replaces the workload's sizes (bf16, same generator) for traffic sweeps.  `--pass bwd`
-times moa_attn_bwd (three launches) on the same workload instead of the forward pass, and
-`--pass qkv` the fused projection moa_qkv_proj producing that workload's Q, K, V from an input
-X [B, N, H*d_k].
+times the backward pass (default workload 2) instead of the forward pass, and `--pass qkv` the
+fused projection moa_qkv_proj producing that workload's Q, K, V from an input X [B, N, H*d_k].
 
 Multi-GPU (torchrun), forward pass: the (b, h) slices of the job are independent problems and
 are partitioned into contiguous ranges, one per rank; each rank runs the forward on its own
@@ -55,6 +54,9 @@ from paper_2606_07713_gb300 import inputs as I  # noqa: E402
 
 METRIC = "attention fwd TFLOP/s and % of GB300 bf16 peak; DRAM bytes vs DNF minimum"
 DEFAULT_WORKLOAD = 5
+# The backward and projection passes default to the d=64 workload: their CPU baselines run the
+# oracle on whole (b, h) slices, which at 32768 x 32768 takes minutes per slice.
+DEFAULT_WORKLOAD_OTHER_PASSES = 2
 PROFILES = {2: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b4h16n2048d64.txt"),
             3: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b2h32n8192d128.txt"),
             4: os.path.join(ROOT, "profiles", "ncu_attn_fwd_bf16_tc_b8h8nq1024nk4096dk128dv64.txt"),
@@ -913,7 +915,9 @@ def main():
     ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference", "classical"], default="ours")
-    ap.add_argument("--workload", type=int, default=DEFAULT_WORKLOAD, choices=sorted(I.CONFIGS))
+    ap.add_argument("--workload", type=int, default=None, choices=sorted(I.CONFIGS),
+                    help=f"workload ID (default: {DEFAULT_WORKLOAD} for the forward pass, "
+                         f"{DEFAULT_WORKLOAD_OTHER_PASSES} for --pass bwd and --pass qkv)")
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle time for the cpu_baseline sample")
     ap.add_argument("--bwd-path", choices=["auto", "fused", "split"], default="auto",
@@ -931,6 +935,8 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.workload is None:
+        args.workload = DEFAULT_WORKLOAD if args.which == "fwd" else DEFAULT_WORKLOAD_OTHER_PASSES
     cfg = I.CONFIGS[args.workload]
     if args.shape:
         dims = [int(t) for t in args.shape.split(",")]

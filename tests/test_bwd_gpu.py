@@ -147,8 +147,8 @@ def test_bwd_fp32_parity(oracle, shape):
 
 
 def test_bwd_bench_workload_sampled_heads(oracle):
-    """The backward on bench.py's default workload (bf16 B=4 H=16 N=2048 d=64, the launch
-    configuration `bench.py --pass bwd` times), two whole (b, h) slices checked against the
+    """The backward on `bench.py --pass bwd`'s default workload (bf16 B=4 H=16 N=2048 d=64, in the
+    launch configuration it times), two whole (b, h) slices checked against the
     oracle element by element (each slice's gradients depend only on that slice)."""
     cfg = I.CONFIGS[2]
     x = I.make_inputs(cfg)
