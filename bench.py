@@ -917,7 +917,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference", "classical"], default="ours")
     ap.add_argument("--workload", type=int, default=None, choices=sorted(I.CONFIGS),
                     help=f"workload ID (default: {DEFAULT_WORKLOAD} for the forward pass, "
-                         f"{DEFAULT_WORKLOAD_OTHER_PASSES} for --pass bwd and --pass qkv)")
+                         f"{DEFAULT_WORKLOAD_OTHER_PASSES} for --pass bwd, --pass qkv and "
+                         f"--impl classical)")
     ap.add_argument("--cpu-budget", type=float, default=12.0,
                     help="seconds of oracle time for the cpu_baseline sample")
     ap.add_argument("--bwd-path", choices=["auto", "fused", "split"], default="auto",
@@ -936,7 +937,9 @@ def main():
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.workload is None:
-        args.workload = DEFAULT_WORKLOAD if args.which == "fwd" else DEFAULT_WORKLOAD_OTHER_PASSES
+        # the classical path materialises N_q x N_k arrays: 34 GB each at workload 5
+        small = args.which != "fwd" or args.impl == "classical"
+        args.workload = DEFAULT_WORKLOAD_OTHER_PASSES if small else DEFAULT_WORKLOAD
     cfg = I.CONFIGS[args.workload]
     if args.shape:
         dims = [int(t) for t in args.shape.split(",")]
