@@ -220,15 +220,17 @@ int moa_qkv_proj(const void* X, const void* W, void* Q, void* K, void* V, int64_
  * problems are independent (Remark in Section 4.2), so the call is pipelined
  * over contiguous ranges of heads (2 to 8 of them, about 16 MiB of inputs each,
  * at most one per (b, h)): the copies of range c+1 into the
- * device run on a library-owned side stream while the kernel of range c runs on
- * `stream`, and each range's output goes back on a second side stream.  Work
- * already queued on `stream` completes before the first copy starts, and
- * `stream` completes only after the last copy back, so hO holds the result once
- * `stream` has been synchronised.  Sizes, layouts, dtype and alignment rules are
- * those of moa_attn_fwd; d* are device pointers owned by the caller, h* host
+ * device run on a library-owned side stream while the kernel of range c runs
+ * (on `stream` for even c, on a library-owned second compute stream for odd c,
+ * so that one range's last wave of CTAs and the next range's first can share the
+ * GPU), and each range's output goes back on a third side stream.  Work
+ * already queued on `stream` completes before the first copy or kernel starts,
+ * and `stream` completes only after the last copy back, so hO holds the result
+ * once `stream` has been synchronised.  Sizes, layouts, dtype and alignment rules
+ * are those of moa_attn_fwd; d* are device pointers owned by the caller, h* host
  * pointers owned by the caller.  Allocates no memory; the first call on a device
- * creates the two side streams and their events (kept until the process exits).
- * Calls on one device enqueue under a lock and share the side streams.
+ * creates the three side streams and their events (kept until the process
+ * exits).  Calls on one device enqueue under a lock and share the side streams.
  */
 int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO, void* dQ,
                         void* dK, void* dV, void* dO, int64_t B, int64_t H, int64_t N_q,

@@ -196,7 +196,9 @@ constexpr int kMaxStageChunks = 8;
 constexpr int64_t kStageChunkBytes = int64_t(16) << 20;
 constexpr int kMaxDevices = 64;
 struct StagePipe {
-  cudaStream_t copy_in = nullptr, copy_out = nullptr;
+  // compute2 takes every other range's kernel, so that the last wave of one range's kernel
+  // shares the GPU with the first CTAs of the next instead of leaving SMs idle.
+  cudaStream_t copy_in = nullptr, copy_out = nullptr, compute2 = nullptr;
   cudaEvent_t start = nullptr, end = nullptr;
   cudaEvent_t in_done[kMaxStageChunks] = {}, kern_done[kMaxStageChunks] = {};
   bool ready = false;
@@ -207,6 +209,7 @@ std::mutex g_pipe_mu[kMaxDevices];
 cudaError_t make_pipe(StagePipe& p) {
   cudaError_t e = cudaStreamCreateWithFlags(&p.copy_in, cudaStreamNonBlocking);
   if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p.copy_out, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p.compute2, cudaStreamNonBlocking);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p.start, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p.end, cudaEventDisableTiming);
   for (int c = 0; e == cudaSuccess && c < kMaxStageChunks; ++c) {
@@ -341,8 +344,9 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
   if (e != cudaSuccess || dev < 0 || dev >= moa::kMaxDevices)
     return moa::fail(MOA_ERR_CUDA, "no usable current device: %s", cudaGetErrorString(e));
   // The (b, h) problems are independent, so the call is pipelined over head ranges: the
-  // host-to-device copies of range c+1 (side stream) overlap the kernel of range c (`stream`),
-  // whose output goes back on a second side stream while later ranges compute.
+  // host-to-device copies of range c+1 (side stream) overlap the kernel of range c (`stream`
+  // for even c, a second compute stream for odd c, so that consecutive kernels may overlap),
+  // whose output goes back on a third side stream while later ranges compute.
   std::lock_guard<std::mutex> lock(moa::g_pipe_mu[dev]);
   moa::StagePipe& p = moa::g_pipes[dev];
   if (!p.ready && (e = moa::make_pipe(p)) != cudaSuccess)
@@ -363,7 +367,8 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
   };
   // Work already queued on `stream` (e.g. a kernel still reading dQ) finishes before the copies.
   if (!chk(cudaEventRecord(p.start, s), "event record") ||
-      !chk(cudaStreamWaitEvent(p.copy_in, p.start, 0), "stream wait"))
+      !chk(cudaStreamWaitEvent(p.copy_in, p.start, 0), "stream wait") ||
+      !chk(cudaStreamWaitEvent(p.compute2, p.start, 0), "stream wait"))
     return MOA_ERR_CUDA;
   for (int c = 0; c < chunks; ++c) {
     const int64_t h0 = c * per, nh = (h0 + per <= BH ? per : BH - h0);
@@ -379,14 +384,15 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
   for (int c = 0; c < chunks; ++c) {
     const int64_t h0 = c * per, nh = (h0 + per <= BH ? per : BH - h0);
     if (nh <= 0) break;
-    if (!chk(cudaStreamWaitEvent(s, p.in_done[c], 0), "stream wait")) return MOA_ERR_CUDA;
+    cudaStream_t cs = (c & 1) ? p.compute2 : s;
+    if (!chk(cudaStreamWaitEvent(cs, p.in_done[c], 0), "stream wait")) return MOA_ERR_CUDA;
     rc = moa::dispatch(static_cast<const char*>(dQ) + h0 * row_bytes[0],
                        static_cast<const char*>(dK) + h0 * row_bytes[1],
                        static_cast<const char*>(dV) + h0 * row_bytes[2],
                        static_cast<char*>(dO) + h0 * row_bytes[3], 1, nh, N_q, N_k, d_k, d_v,
-                       scale, dtype, stream);
+                       scale, dtype, cs);
     if (rc != MOA_OK) return rc;
-    if (!chk(cudaEventRecord(p.kern_done[c], s), "event record") ||
+    if (!chk(cudaEventRecord(p.kern_done[c], cs), "event record") ||
         !chk(cudaStreamWaitEvent(p.copy_out, p.kern_done[c], 0), "stream wait") ||
         !chk(cudaMemcpyAsync(static_cast<char*>(hO) + h0 * row_bytes[3],
                              static_cast<const char*>(dO) + h0 * row_bytes[3],
@@ -394,7 +400,8 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
              "device-to-host copy"))
       return MOA_ERR_CUDA;
   }
-  // `stream` completes only after the last copy back: synchronising it makes hO valid.
+  // `stream` completes only after the last copy back, which follows every range's kernel on
+  // either compute stream: synchronising `stream` makes hO valid.
   if (!chk(cudaEventRecord(p.end, p.copy_out), "event record") ||
       !chk(cudaStreamWaitEvent(s, p.end, 0), "stream wait"))
     return MOA_ERR_CUDA;
