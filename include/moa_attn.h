@@ -218,8 +218,9 @@ int moa_qkv_proj(const void* X, const void* W, void* Q, void* K, void* V, int64_
  * hV (host memory, ideally page-locked) into the caller's device buffers dQ,
  * dK, dV, runs the attention on them and copies dO back into hO.  The (b, h)
  * problems are independent (Remark in Section 4.2), so the call is pipelined
- * over contiguous ranges of heads (2 to 8 of them, about 16 MiB of inputs each,
- * at most one per (b, h)): the copies of range c+1 into the
+ * over contiguous ranges of heads (2 to 8 of them, about 16 MiB of inputs each
+ * on average, the first and last ones smaller, at least one (b, h) each): the
+ * copies of range c+1 into the
  * device run on a library-owned side stream while the kernel of range c runs
  * (on `stream` for even c, on a library-owned second compute stream for odd c,
  * so that one range's last wave of CTAs and the next range's first can share the

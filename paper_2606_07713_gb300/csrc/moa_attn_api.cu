@@ -187,13 +187,39 @@ int dispatch(const void* Q, const void* K, const void* V, void* O, int64_t B, in
 // Side streams and events of the pipelined staged call, one set per device, created on the
 // device's first staged call.  The mutex is held while a call enqueues its work, so the events
 // of two concurrent calls never interleave.
-// Head ranges of the staged call: about kStageChunkBytes of inputs each, 2 to kMaxStageChunks
-// of them (measured on a GB300: 4x16x2048^2 d=64, 50 MB of inputs, is fastest with 4 ranges,
-// 191 TFLOP/s end to end vs 183 with 2 and 173 with 8; 2x32x8192^2 d=128, 403 MB, with 6 to 8,
-// 905 vs 830 with 4: more ranges shorten the pipeline's fill and drain, smaller ones copy less
-// efficiently).
+// Head ranges of the staged call: about kStageChunkBytes of inputs on average, 2 to
+// kMaxStageChunks of them, the outer ones smaller (measured on a GB300, end to end, with kernels
+// on two compute streams: equal ranges / weights 1, 2, 3, 3, ..., 3, 2, 1 gave 185 / 201 TFLOP/s
+// on 4x16x2048^2 d=64, 912 / 955 on 2x32x8192^2 d=128, 1630 / 1678 on 1x16x32768^2 d=128; up to
+// 16 ranges, 8 MiB ranges or weights capped at 2 or 4 were no better).
 constexpr int kMaxStageChunks = 8;
 constexpr int64_t kStageChunkBytes = int64_t(16) << 20;
+// Range sizes: 0 = equal; R > 0 = weights min(c + 1, n - c, R), so that the first range (whose
+// copy nothing hides) and the last (whose kernel and copy back nothing hides) are small.
+constexpr int kStageRamp = 3;
+
+// Head boundaries of the staged call's ranges: range c is [bound[c], bound[c + 1]).
+void stage_bounds(int64_t BH, int chunks, int64_t* bound) {
+  bound[0] = 0;
+  if (kStageRamp <= 0) {
+    const int64_t per = (BH + chunks - 1) / chunks;
+    for (int c = 1; c <= chunks; ++c) bound[c] = c * per < BH ? c * per : BH;
+    return;
+  }
+  int64_t w[kMaxStageChunks + 1], total = 0;
+  for (int c = 0; c < chunks; ++c) {
+    int64_t x = c + 1 < chunks - c ? c + 1 : chunks - c;
+    w[c] = x < kStageRamp ? x : kStageRamp;
+    total += w[c];
+  }
+  int64_t acc = 0;
+  for (int c = 0; c < chunks; ++c) {
+    acc += w[c];
+    int64_t b = (BH * acc + total / 2) / total;
+    const int64_t lo = bound[c] + 1, hi = BH - (chunks - 1 - c);  // at least one head each
+    bound[c + 1] = b < lo ? lo : (b > hi ? hi : b);
+  }
+}
 constexpr int kMaxDevices = 64;
 struct StagePipe {
   // compute2 takes every other range's kernel, so that the last wave of one range's kernel
@@ -358,7 +384,8 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
   int64_t want = (in_bytes + moa::kStageChunkBytes - 1) / moa::kStageChunkBytes;
   want = want < 2 ? 2 : (want > moa::kMaxStageChunks ? moa::kMaxStageChunks : want);
   const int chunks = int(BH < want ? BH : want);
-  const int64_t per = (BH + chunks - 1) / chunks;
+  int64_t bound[moa::kMaxStageChunks + 1];
+  moa::stage_bounds(BH, chunks, bound);
   const void* src[3] = {hQ, hK, hV};
   void* dst[3] = {dQ, dK, dV};
   auto chk = [&](cudaError_t err, const char* what) {
@@ -371,7 +398,7 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
       !chk(cudaStreamWaitEvent(p.compute2, p.start, 0), "stream wait"))
     return MOA_ERR_CUDA;
   for (int c = 0; c < chunks; ++c) {
-    const int64_t h0 = c * per, nh = (h0 + per <= BH ? per : BH - h0);
+    const int64_t h0 = bound[c], nh = bound[c + 1] - bound[c];
     if (nh <= 0) break;
     for (int t = 0; t < 3; ++t)
       if (!chk(cudaMemcpyAsync(static_cast<char*>(dst[t]) + h0 * row_bytes[t],
@@ -382,7 +409,7 @@ int moa_attn_fwd_staged(const void* hQ, const void* hK, const void* hV, void* hO
     if (!chk(cudaEventRecord(p.in_done[c], p.copy_in), "event record")) return MOA_ERR_CUDA;
   }
   for (int c = 0; c < chunks; ++c) {
-    const int64_t h0 = c * per, nh = (h0 + per <= BH ? per : BH - h0);
+    const int64_t h0 = bound[c], nh = bound[c + 1] - bound[c];
     if (nh <= 0) break;
     cudaStream_t cs = (c & 1) ? p.compute2 : s;
     if (!chk(cudaStreamWaitEvent(cs, p.in_done[c], 0), "stream wait")) return MOA_ERR_CUDA;

@@ -140,6 +140,26 @@ def test_staged_api_matches_device_api():
     assert torch.equal(ho, o.cpu())
 
 
+@pytest.mark.parametrize("shape", [(4, 16, 4096, 4096, 64, 64), (1, 11, 8000, 16000, 128, 128)])
+def test_staged_many_ranges_matches_device_api(shape):
+    """Inputs of about 100 MB: six or seven head ranges of unequal size (the outer ones
+    smallest), kernels alternating between two streams.  The host output must hold the bits of
+    the device call's output for every head."""
+    B, H, Nq, Nk, dk, dv = shape
+    g = torch.Generator(device="cuda").manual_seed(61)
+    q = torch.randn((B, H, Nq, dk), generator=g, device="cuda").to(torch.bfloat16)
+    k = torch.randn((B, H, Nk, dk), generator=g, device="cuda").to(torch.bfloat16)
+    v = torch.randn((B, H, Nk, dv), generator=g, device="cuda").to(torch.bfloat16)
+    o = pkg.attn_fwd(q, k, v)
+    hq, hk, hv = (t.cpu().pin_memory() for t in (q, k, v))
+    ho = torch.full(o.shape, float("nan"), dtype=o.dtype).pin_memory()
+    dq, dk_, dv_ = (torch.empty_like(t) for t in (q, k, v))
+    do = torch.empty_like(o)
+    pkg.attn_fwd_staged(hq, hk, hv, ho, dq, dk_, dv_, do)
+    torch.cuda.synchronize()
+    assert torch.equal(ho, o.cpu())
+
+
 def test_device_status_clean_after_runs():
     x = inputs((1, 1, 128, 128, 64, 64), 13)
     pkg.attn_fwd(*to_device(x))
