@@ -408,6 +408,10 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
                 "peak_source": f"{peak_src} bf16_tflops (burst; kernel timed alone)",
                 "unit": "TFLOP/s",
                 "frac": round(achieved / peak, 4) if peak else None,
+                # the same against the GEMM peak measured back to back under the power cap,
+                # the other denominator for a kernel timed inside a long loop
+                "frac_of_sustained": (round(achieved / float(peaks["bf16_tflops_sustained"]), 4)
+                                      if peak and peaks.get("bf16_tflops_sustained") else None),
                 **tr,
                 "traffic_source": (os.path.relpath(PROFILES[cfg.cfg_id], ROOT)
                                    if tr["traffic"] is not None else
