@@ -15,9 +15,8 @@
 //     rescaled by exp2(m_old - m_new); otherwise the stale m is kept.  Both are exact: O and l
 //     always share the same reference maximum, and exponentials stay <= 2^kRescaleLog2.
 //   * The unnormalised probabilities P are rounded to bf16 and stored where the second
-//     tensor-core product O += P V (Eq. output_dnf) reads them: TMEM columns of their own
-//     (d_v = 64) or a 32 KB shared-memory tile per Q tile (d_v = 128, where S and O fill the
-//     TMEM).  V is the "MN-major" B operand, again as stored.
+//     tensor-core product O += P V (Eq. output_dnf) reads them: TMEM columns of their own, the
+//     A operand of that product.  V is the "MN-major" B operand, again as stored.
 //   * Step IV (division, Section 4.5) is applied once per row in the epilogue: O / l.
 //
 // CTA organisation, two-tile kernel (one CTA per SM: 512 TMEM columns, up to ~225 KB shared
@@ -31,13 +30,13 @@
 // One-tile kernel (d_k = d_v = 64 without a split key axis; two CTAs per SM, 256 TMEM columns
 // and ~98 KB of shared memory each): work item = (b*H + h, block of 128 query rows); warps 0-3
 // softmax + epilogue, warp 4 TMEM allocation and tcgen05.mma, warp 5 TMA loads.
-// K and V tiles of 128 keys stream through an NS-stage shared-memory ring.  One schedule: P_j
-// has a buffer of its own (TMEM S0 S1 P0 P1 O0 O1 at d_v = 64, one tile: S0 P0 O0; TMEM
-// S0 S1 O0 O1 plus P0 P1 in shared memory at d_v = 128).  As soon as the softmax has read
-// S_j(n) into registers, tile j's issuing thread computes S_j(n+1), and it runs
-// O_j += P_j(n) V(n) once P_j(n) is written, so the softmax never waits for the product with
-// V; ring order K0 K1 V0 K2 V1 ...
-// TMEM lane = row of the Q tile.
+// K and V tiles of 128 keys stream through an NS-stage shared-memory ring, in the order the
+// products use them: K0 K1 V0 K2 V1 ...  TMEM columns: S0 S1 P0 P1 O0 O1 at d_v = 64; one S
+// buffer shared by the two tiles, S P0 P1 O0 O1, at d_v = 128 (the two O take 256 columns);
+// one tile: S0 P0 O0.  As soon as the S buffer's last reader holds S_j(n) in registers, tile
+// j's issuing thread computes S_j(n+1); it runs O_j += P_j(n) V(n) once P_j(n) is written.  The
+// softmax writes P_j(n) once O_j += P_j(n-1) V(n-1) is done (it computes the first chunks of
+// exponentials before waiting for that).  TMEM lane = row of the Q tile.
 
 // Every mbarrier wait is bounded (globaltimer); on expiry the kernel records
 // MOA_ERR_DEVICE_TIMEOUT in g_moa_bf16_status, makes every role leave its loop, and still
@@ -445,8 +444,8 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
           rescale = true;
         }
       }
-      // Step II + III: p = exp2(c*s - m), row sum, P -> bf16 pairs into the S columns (chunk c
-      // of 32 scores becomes 16 packed columns at column 16c; all of S is already in registers).
+      // Step II + III: p = exp2(c*s - m), row sum, P -> bf16 pairs into P_j's TMEM columns
+      // (chunk c of 32 scores becomes 16 packed columns at column 16c of P_j).
       const uint64_t cc = pack_f32x2(c_log2, c_log2);
       const uint64_t mm = pack_f32x2(-m, -m);
       float l0 = 0.f, l1 = 0.f, l2 = 0.f, l3 = 0.f;
