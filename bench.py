@@ -364,7 +364,8 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
     barrier()
     sampler.mark(t0, time.time())
     clocks = sampler.stop()
-    e2e_ms = float(np.sum([a.elapsed_time(b) for a, b in ev2]))
+    e2e_step_ms = [a.elapsed_time(b) for a, b in ev2]
+    e2e_ms = float(np.sum(e2e_step_ms))
     pkg.check(pkg.get_device_status())
 
     total_ms, e2e_ms = reduce_max_over_ranks([total_ms, e2e_ms], device=dev)
@@ -426,6 +427,9 @@ def run_ours(args, cfg: I.AttnConfig) -> None:
                 "h2d_bytes_per_step": int(in_bytes * copies),
                 "d2h_bytes_per_step": int(out_bytes * copies),
                 "api": "moa_attn_fwd_staged",
+                # rank 0's steps: the value above sums all of them, slow outliers included
+                "ms_median": round(float(np.median(e2e_step_ms)), 6),
+                "ms_max": round(float(np.max(e2e_step_ms)), 6),
             },
             # one kernel per step on every rank that owns at least one slice
             "gpu_launches": args.steps * min(world, job_slices),
