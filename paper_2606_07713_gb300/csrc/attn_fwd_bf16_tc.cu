@@ -26,7 +26,8 @@
 //              (thread t of such a warpgroup owns query row t of its tile);
 //   warp 8:    TMEM allocation; issues the tcgen05.mma products of Q tile 0;
 //   warp 9:    the single thread that issues all TMA loads;
-//   warp 10:   issues the tcgen05.mma products of Q tile 1.
+//   warp 10:   issues the tcgen05.mma products of Q tile 1;
+//   warp 11:   idle (it completes warps 8-11 as one warpgroup for the register split).
 // One-tile kernel (d_k = d_v = 64 without a split key axis; two CTAs per SM, 256 TMEM columns
 // and ~98 KB of shared memory each): work item = (b*H + h, block of 128 query rows); warps 0-3
 // softmax + epilogue, warp 4 TMEM allocation and tcgen05.mma, warp 5 TMA loads.
@@ -45,6 +46,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstdio>
 #include <mutex>
@@ -79,11 +81,23 @@ struct Cfg {
   // Warps: 4 softmax warps per Q tile, then the MMA warp of tile 0 (it also allocates and frees
   // TMEM), the TMA warp and, with two tiles, the MMA warp of tile 1.  One-tile CTAs run two per
   // SM (half the registers, TMEM and shared memory each).
-  static constexpr int kThreads = QT == 2 ? 352 : 192;
+  static constexpr int kThreads = QT == 2 ? 384 : 192;
   static constexpr int kMinBlocks = QT == 2 ? 1 : 2;
   static constexpr int kMmaWarp0 = 4 * QT;
   static constexpr int kLoadWarp = 4 * QT + 1;
   static constexpr int kMmaWarp1 = QT == 2 ? 10 : -1;
+  // Two tiles: warps 8-11 (MMA issuer of tile 0, TMA, MMA issuer of tile 1, one idle warp) form
+  // one warpgroup whose registers move to the two softmax warpgroups with setmaxnreg.  Launched
+  // with kRegsLaunch per thread; 256 * kRegsSoftmax + 128 * kRegsCtrl equals the launch
+  // allocation, so the softmax warps never wait for registers the CTA does not hold (the host
+  // checks the compiled count), and each scheduler's two softmax warps and one control warp fit
+  // its 16K registers.  Measured +1.1 to +2 % on 2x32x8192^2, 1x16x32768^2 and
+  // 8x8x1024x4096 against 11 warps at 168 registers each (216/56 the same; 4 early chunks no
+  // better).
+  static constexpr bool kRegSplit = QT == 2;
+  static constexpr int kRegsLaunch = 168, kRegsSoftmax = 208, kRegsCtrl = 88;
+  static_assert(!kRegSplit || 256 * kRegsSoftmax + 128 * kRegsCtrl <= kThreads * kRegsLaunch,
+                "register split");
   static constexpr int kTmemCols = 256 * QT;
   static_assert(DV == 64 || DV == 128, "d_v must be 64 or 128");
   // One 128-byte swizzle panel holds 64 bf16 columns of 128 rows: 16 KB.
@@ -240,6 +254,10 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
   tc_fence_after_sync();
   const uint32_t tmem = *tmem_slot;
 
+  if (warp >= 4 * QT) {
+    // Control warps (MMA issuers, TMA producer, and with two tiles an idle warp).
+    if constexpr (C::kRegSplit)
+      asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(C::kRegsCtrl));
   if (warp == kLoadWarp) {
     // ---------------------------------------------------------------- TMA producer
     if (lane == 0) {
@@ -392,7 +410,10 @@ attn_fwd_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
       // TMEM is quiescent before it is freed even on the abort path.
       mma_commit(o_done(j));
     }
+  }
   } else {
+    if constexpr (C::kRegSplit)
+      asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(C::kRegsSoftmax));
     // ---------------------------------------------------------------- softmax warpgroups
     const int j = warp >> 2;                // Q tile of this warpgroup
     const int lane_base = (warp & 3) * 32;  // TMEM lanes of this warp
@@ -722,6 +743,27 @@ int launch_tc(const AttnArgs& a, const CUtensorMap& mq, const CUtensorMap& mk,
   if (attr_err != cudaSuccess) {
     snprintf(msg, msglen, "cudaFuncSetAttribute (bf16 kernel): %s", cudaGetErrorString(attr_err));
     return 5;
+  }
+  if (split || QT1 == 2) {
+    // The register split of the two-tile kernel moves registers inside the CTA's launch
+    // allocation: refuse a build whose allocation is short of the split's sum.
+    static std::atomic<int> regs_of[2] = {-1, -1};  // unsplit and split instance
+    std::atomic<int>& regs = regs_of[split ? 1 : 0];
+    if (regs.load(std::memory_order_relaxed) < 0) {
+      cudaFuncAttributes fa;
+      const cudaError_t e = cudaFuncGetAttributes(&fa, reinterpret_cast<const void*>(kern));
+      if (e != cudaSuccess) {
+        snprintf(msg, msglen, "cudaFuncGetAttributes (bf16 kernel): %s", cudaGetErrorString(e));
+        return 5;
+      }
+      regs.store(fa.numRegs, std::memory_order_relaxed);
+    }
+    const int r = regs.load(std::memory_order_relaxed);
+    if (r * C::kThreads < 256 * C::kRegsSoftmax + 128 * C::kRegsCtrl) {
+      snprintf(msg, msglen, "bf16 kernel compiled to %d registers per thread, short of the "
+               "register split", r);
+      return 5;
+    }
   }
   const int64_t n_qblocks = (a.Nq + tile_rows - 1) / tile_rows;
   const int64_t grid = a.B * a.H * n_qblocks * sp.n_splits;
