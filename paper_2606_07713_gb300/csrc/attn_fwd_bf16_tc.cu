@@ -125,9 +125,10 @@ struct Cfg {
   static constexpr int kIssuers = QT;
   // Chunks of 32 exponentials computed before the wait for P's buffer (the rest after it), so
   // that the wait for the previous block's P V overlaps them (measured on 4x16x2048^2, d=64:
-  // 0 -> 2 chunks 740 -> 812 TFLOP/s; 1x16x32768^2, d=128: 0 -> 3 chunks +2 %; more chunks
-  // spill registers and run slower).
-  static constexpr int kEarlyChunks = QT == 1 ? 2 : DV == 64 ? 0 : 3;
+  // 0 -> 2 chunks 740 -> 812 TFLOP/s; 1x16x32768^2, d=128: 0 -> 3 chunks +2 %; with the
+  // two-tile register split, 8x8x1024x4096 (d_k=128, d_v=64): 0 -> 2 chunks 1064 -> 1087, 3 no
+  // better; more chunks than these spill or gain nothing).
+  static constexpr int kEarlyChunks = QT == 1 ? 2 : DV == 64 ? 2 : 3;
   // barriers: full[NS], empty[NS], q_full, s_full[2], p_ready[2], o_done[2], s_free[2], p_free[2]
   static constexpr int kNumBars = 2 * kStages + 11;
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem base, abort flag
